@@ -1,0 +1,351 @@
+#!/usr/bin/env python
+"""Throughput of the BACON end-of-prefill KV-cache compression step.
+
+One step = the whole path (window scores, calibration, top-B selection,
+compaction) for every layer and kv-head of one batch of synthetic prompts,
+through the C-ABI call ``bacon_compress_all_layers`` with the inputs already
+resident in HBM.  Default workload: the long GUI/screenshot shape (28 layers,
+28 query / 4 kv heads, head_dim 128, 16384-token prompts, window 64, pool 7,
+budget 1024, 4 requests).  Inputs (1.9 GB of K per step) are far larger than
+L2, so no flush is needed between steps.
+
+Prints one JSON line.  ``--impl reference`` times the CPU oracle instead
+(bounded sample of the same workload on the host cores).
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "layer-heads compressed/s"
+UNIT = "layer-heads/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("bacon", "reference"), default="bacon")
+    ap.add_argument("--config", default="gui")
+    ap.add_argument("--budget", type=int, default=None)
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, "fallback"
+
+
+def config_dict(wl, budget, n_gpus):
+    return {"workload": f"{wl.name}: {wl.layers} layers, {wl.q_heads}/{wl.kv_heads} heads, "
+                        f"d {wl.head_dim}, N {wl.seq_len}, W {wl.window}, pool {wl.pool}, "
+                        f"budget {budget}, {wl.requests} requests",
+            "requests_per_gpu": wl.requests, "seq_len": wl.seq_len, "layers": wl.layers,
+            "q_heads": wl.q_heads, "kv_heads": wl.kv_heads, "head_dim": wl.head_dim,
+            "window": wl.window, "budget": budget,
+            "parallelism": f"replicas x{n_gpus} (independent requests per GPU)",
+            "l2": "inputs larger than L2 (K alone %.2f GB per step)" %
+                  (wl.requests * wl.layers * wl.kv_heads * wl.seq_len * wl.head_dim * 2 / 1e9)}
+
+
+# ------------------------------------------------------------- clocks
+
+class ClockSampler:
+    FIELDS = ("uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid: str | None):
+        self.uuid = uuid
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                if self.uuid and self.uuid not in parts[0]:
+                    continue
+                rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "", 1).isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "", 1).isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+
+
+# --------------------------------------------------------- traffic
+
+def kernel_traffic(kernel: str):
+    """DRAM bytes per launch from the committed ncu summary, or None when the
+    kernel's source changed since the counters were taken."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)[kernel]
+        src = os.path.join(ROOT, "paper_2606_14782_gb300", "csrc", rec["source"])
+        digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        if digest != rec["source_sha256_16"]:
+            return None
+        return float(rec["dram_bytes_per_launch"])
+    except Exception:
+        return None
+
+
+# ---------------------------------------------------- CPU oracle legs
+
+def oracle_sample(wl, budget, units, threads):
+    """Time the CPU oracle on `units` of a same-shaped host workload."""
+    import oracle
+    from paper_2606_14782_gb300 import workloads
+
+    layers_needed = max(l for _, l, _ in units) + 1
+    host = workloads.generate(wl.with_(layers=layers_needed), seed=0, device="cpu")
+    qb, kb, vb = (workloads.bf16_bits(t) for t in (host.qwin, host.k, host.v))
+    p = oracle.Params(pool_kernel=wl.pool)
+    t0 = time.perf_counter()
+    oracle.compress(qb, kb, vb, budget, p, threads=threads, units=units)
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(wl, budget):
+    threads = min(os.cpu_count() or 1, wl.requests * wl.kv_heads)
+    units = [(r, 0, h) for r in range(wl.requests) for h in range(wl.kv_heads)]
+    secs = oracle_sample(wl, budget, units, threads)
+    return {"value": len(units) / secs, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": f"{len(units)} layer-heads (layer 0 of every request and kv-head) of the "
+                      f"same workload, double precision, {threads} threads, {secs:.1f} s"}
+
+
+def run_reference(args):
+    from paper_2606_14782_gb300 import workloads
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    wl = workloads.CONFIGS[args.config]
+    budget = args.budget or max(wl.budgets)
+    threads = min(os.cpu_count() or 1, wl.requests * wl.kv_heads)
+    units = [(r, 0, h) for r in range(wl.requests) for h in range(wl.kv_heads)]
+    # one step: layer 0 of every (request, kv-head) of the workload
+    import oracle
+    host = workloads.generate(wl.with_(layers=1), seed=0, device="cpu")
+    qb, kb, vb = (workloads.bf16_bits(t) for t in (host.qwin, host.k, host.v))
+    p = oracle.Params(pool_kernel=wl.pool)
+    for _ in range(args.warmup):
+        oracle.compress(qb, kb, vb, budget, p, threads=threads, units=units)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.compress(qb, kb, vb, budget, p, threads=threads, units=units)
+    secs = time.perf_counter() - t0
+    value = len(units) * args.steps / secs
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": 0, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "impl": "reference",
+            "config": config_dict(wl, budget, 1),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                             "sample": f"each step: {len(units)} layer-heads (layer 0 of every "
+                                       "request and kv-head), double precision"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------ GPU arm
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+        return
+    import torch
+    import torch.distributed as dist
+
+    from paper_2606_14782_gb300 import bacon, workloads
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    wl = workloads.CONFIGS[args.config]
+    budget = args.budget or max(wl.budgets)
+    x = workloads.generate(wl, seed=rank, device=dev)
+    p = bacon.default_params(max_seq_len=wl.seq_len, max_requests=wl.requests)
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool,
+                        budget, params=p)
+    ko, vo, idx = ctx.compress_all_layers(x.qwin, x.k, x.v, budget)
+    stream = torch.cuda.current_stream()
+    for _ in range(max(3, args.warmup)):
+        ctx.compress_all_layers(x.qwin, x.k, x.v, budget, ko, vo, idx)
+    ctx.sync()
+
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        pass
+    sampler = ClockSampler(uuid)
+    sampler.start()
+    time.sleep(0.3)
+    ctx.profile(True)
+    ctx.profile_read()
+    barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        ctx.compress_all_layers(x.qwin, x.k, x.v, budget, ko, vo, idx)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clocks = sampler.stop()
+    prof = ctx.profile_read()
+    ctx.profile(False)
+    ctx.sync()
+    ms = e0.elapsed_time(e1) / args.steps
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+
+    units = wl.requests * wl.layers * wl.kv_heads
+    value = world * units / (ms / 1e3)
+    hbm, tflops, peak_src = peaks()
+
+    # per-kernel times measured live (CUDA events around each launch)
+    K_bytes = wl.requests * wl.layers * wl.kv_heads * wl.seq_len * wl.head_dim * 2
+    Q_bytes = wl.requests * wl.layers * wl.q_heads * wl.window * wl.head_dim * 2
+    tok = wl.requests * wl.layers * wl.kv_heads * wl.seq_len
+    kept = min(budget, wl.seq_len)
+    algo_bytes = {
+        "window_stats": K_bytes + Q_bytes,
+        "window_scores": K_bytes + Q_bytes + 12 * tok,
+        "window_combine": 0,
+        "calibrate_select": tok * (4 + 4 * (1 + min(4, wl.layers - 1))) + units * kept * 4,
+        "gather": 4 * units * kept * wl.head_dim * 2 + units * kept * 4,
+    }
+    total = sum(t for t, _ in prof.values())
+    kernels = {k: {"ms_per_launch": (t / n if n else None), "share": (t / total if total else None)}
+               for k, (t, n) in prof.items()}
+    dom = max(prof, key=lambda k: prof[k][0])
+    dom_ms = prof[dom][0] / max(1, prof[dom][1])
+    achieved = algo_bytes[dom] / (dom_ms / 1e3) / 1e9
+    flops = 2 * wl.requests * wl.layers * wl.q_heads * wl.window * wl.seq_len * wl.head_dim
+    traffic = kernel_traffic(dom)
+    roofline = {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm,
+                "unit": "GB/s", "frac": achieved / hbm, "peak_source": peak_src,
+                "traffic": traffic,
+                "algorithmic_bytes_per_launch": algo_bytes[dom],
+                "tensor_tflops_one_pass": (flops / (dom_ms / 1e3) / 1e12
+                                           if dom.startswith("window") else None)}
+    step_bytes = wl.bytes_model(budget)
+
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "ms_per_request": ms / wl.requests,
+            "achieved_step_gbs": step_bytes / (ms / 1e3) / 1e9,
+            "step_roofline_frac": step_bytes / (ms / 1e3) / 1e9 / hbm,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded, paper-shaped; no datasets)",
+            "config": config_dict(wl, budget, world),
+            "gpu_launches": 5 * args.steps, "roofline": roofline, "kernels": kernels,
+            "clocks": clocks}
+
+    # end to end through the host-buffer C call: H2D inputs, compress, D2H outputs
+    if not args.no_e2e:
+        del x
+        torch.cuda.empty_cache()
+        hx = workloads.generate(wl, seed=rank, device=dev)
+        hq, hk, hv = (t.cpu().pin_memory() for t in (hx.qwin, hx.k, hx.v))
+        del hx
+        torch.cuda.empty_cache()
+        shape_o = (wl.requests, wl.layers, wl.kv_heads, kept, wl.head_dim)
+        hko = torch.empty(shape_o, dtype=torch.bfloat16, pin_memory=True)
+        hvo = torch.empty(shape_o, dtype=torch.bfloat16, pin_memory=True)
+        hidx = torch.empty(shape_o[:-1], dtype=torch.int32, pin_memory=True)
+        ctx.compress_host(hq, hk, hv, budget, hko, hvo, hidx)
+        barrier()
+        torch.cuda.synchronize()
+        f0 = torch.cuda.Event(enable_timing=True)
+        f1 = torch.cuda.Event(enable_timing=True)
+        f0.record(stream)
+        for _ in range(args.e2e_steps):
+            ctx.compress_host(hq, hk, hv, budget, hko, hvo, hidx)
+        f1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = f0.elapsed_time(f1) / args.e2e_steps
+        if world > 1:
+            t = torch.tensor([e2e_ms], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_ms = float(t.item())
+        h2d = sum(t.numel() * t.element_size() for t in (hq, hk, hv))
+        d2h = sum(t.numel() * t.element_size() for t in (hko, hvo, hidx))
+        line["e2e"] = {"value": world * units / (e2e_ms / 1e3), "unit": UNIT,
+                       "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d,
+                       "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
+                       "path": "bacon_compress_host (pinned host buffers)"}
+    ctx.close()
+
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, budget)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,715 @@
+// C ABI of the BACON library: argument checks, context and state ownership,
+// and the launch sequence of the compression step.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "../../include/bacon.h"
+#include "common.cuh"
+
+using namespace bacon;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+bacon_status fail(bacon_status st, const char* fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return st;
+}
+
+bacon_status cuda_fail(cudaError_t e, const char* what)
+{
+    return fail(BACON_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define BACON_CUDA(call, what)                         \
+    do {                                               \
+        cudaError_t e_ = (call);                       \
+        if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+    } while (0)
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+constexpr int kChunkTokens = 1024;  // pass-1 token chunk (multiple of the 128-token tile)
+constexpr int kMaxSeq = 24576;      // calibration keeps 2 x N fp32 in shared memory
+
+// Makes the context's device current for the duration of a call.
+struct DeviceGuard {
+    int prev = -1;
+    bool ok = true;
+    explicit DeviceGuard(int dev)
+    {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        if (prev != dev) ok = cudaSetDevice(dev) == cudaSuccess;
+    }
+    ~DeviceGuard()
+    {
+        int cur = -1;
+        if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+    }
+};
+
+template <typename T>
+cudaError_t dalloc(T** p, size_t count)
+{
+    *p = nullptr;
+    if (count == 0) return cudaSuccess;
+    return cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T));
+}
+
+}  // namespace
+
+struct bacon_ctx {
+    int device = 0;
+    int layers = 0, hkv = 0, hq = 0, group = 0, d = 0, W = 0, pool = 1, budget = 0;
+    int rows = 0;
+    bacon_params p{};
+    int max_chunks = 0;
+    size_t unit_cap = 0;  // max_requests * layers * hkv
+    float* B = nullptr;
+    float* Q = nullptr;
+    float* E = nullptr;
+    float* S = nullptr;
+    float* V = nullptr;
+    float* Bp = nullptr;
+    float* lam = nullptr;
+    float* lse2 = nullptr;
+    float2* partial = nullptr;
+    int* err = nullptr;
+    int last_units = 0, last_N = 0;
+    // staging buffers of bacon_compress_host
+    void* hq_buf = nullptr;
+    void* hk_buf = nullptr;
+    void* hv_buf = nullptr;
+    void* hko_buf = nullptr;
+    void* hvo_buf = nullptr;
+    int32_t* hidx_buf = nullptr;
+    size_t hq_cap = 0, hkv_cap = 0, hout_cap = 0, hidx_cap = 0;
+    // per-kernel timing (bacon_profile_enable)
+    int prof_on = 0;
+    std::vector<cudaEvent_t> ev_free;
+    std::vector<std::vector<cudaEvent_t>> ev_pending;  // 6 events per call
+};
+
+struct bacon_state {
+    bacon_ctx* ctx = nullptr;
+    int next_layer = 0;
+    int N = 0;
+    int scored = 0;
+    int ring = 1;
+    float* Ering = nullptr;  // [ring][hkv][max_seq_len]
+    float* B = nullptr;
+    float* Q = nullptr;
+    float* S = nullptr;
+    float* lam = nullptr;
+    float* lse2 = nullptr;
+    float2* partial = nullptr;
+};
+
+namespace {
+
+Calib calib_of(const bacon_ctx* c)
+{
+    Calib k;
+    k.r = c->p.r;
+    k.m = c->p.m;
+    k.rho = c->p.rho;
+    k.gamma = c->p.gamma;
+    k.eps = c->p.eps;
+    k.use_E = c->p.use_E;
+    k.use_L = c->p.use_L;
+    k.use_T = c->p.use_T;
+    k.keep_window = c->p.keep_window;
+    k.pool = c->pool;
+    return k;
+}
+
+Shape shape_of(const bacon_ctx* c, int layers, int requests, int N)
+{
+    Shape s;
+    s.layers = layers;
+    s.hkv = c->hkv;
+    s.group = c->group;
+    s.d = c->d;
+    s.W = c->W;
+    s.N = N;
+    s.units = requests * layers * c->hkv;
+    s.rows = c->rows;
+    return s;
+}
+
+bacon_status check_seq(const bacon_ctx* c, int N, int budget)
+{
+    if (N < c->W) return fail(BACON_EINVAL, "seq_len %d is shorter than the window %d", N, c->W);
+    if (N > c->p.max_seq_len)
+        return fail(BACON_EINVAL, "seq_len %d exceeds max_seq_len %d", N, c->p.max_seq_len);
+    if (budget < 1) return fail(BACON_EINVAL, "budget must be positive");
+    if (c->p.keep_window && budget < c->W)
+        return fail(BACON_EINVAL, "budget %d is smaller than the window %d", budget, c->W);
+    return BACON_OK;
+}
+
+// Eqs. 1, 2, 4 for every unit of the call: B, Q and E (E written to `E`).
+bacon_status run_window(const QKTable& tab, const Shape& s, float2* partial, float* lse2,
+                        float* B, float* Q, float* E, cudaStream_t st)
+{
+    const int chunks = (s.N + kChunkTokens - 1) / kChunkTokens;
+    BACON_CUDA(launch_window_stats(tab, s, kChunkTokens, partial, st), "window_stats launch");
+    BACON_CUDA(launch_window_combine(s, chunks, partial, lse2, st), "window_combine launch");
+    BACON_CUDA(launch_window_scores(tab, s, lse2, B, Q, E, st), "window_scores launch");
+    return BACON_OK;
+}
+
+void free_ctx_buffers(bacon_ctx* c)
+{
+    for (auto& v : c->ev_pending)
+        for (cudaEvent_t e : v)
+            if (e) cudaEventDestroy(e);
+    for (cudaEvent_t e : c->ev_free)
+        if (e) cudaEventDestroy(e);
+    c->ev_pending.clear();
+    c->ev_free.clear();
+    void* bufs[] = {c->B,      c->Q,      c->E,      c->S,      c->V,      c->Bp,
+                    c->lam,    c->lse2,   c->partial, c->err,   c->hq_buf, c->hk_buf,
+                    c->hv_buf, c->hko_buf, c->hvo_buf, c->hidx_buf};
+    for (void* b : bufs)
+        if (b) cudaFree(b);
+}
+
+// Events bracketing the five launches of one call (profiling only).
+struct StageEvents {
+    bacon_ctx* c;
+    cudaStream_t st;
+    std::vector<cudaEvent_t> ev;
+    StageEvents(bacon_ctx* c_, cudaStream_t st_) : c(c_), st(st_)
+    {
+        if (!c->prof_on) return;
+        for (int i = 0; i < BACON_PROFILE_STAGES + 1; ++i) {
+            cudaEvent_t e = nullptr;
+            if (!c->ev_free.empty()) {
+                e = c->ev_free.back();
+                c->ev_free.pop_back();
+            } else if (cudaEventCreate(&e) != cudaSuccess) {
+                e = nullptr;
+            }
+            ev.push_back(e);
+        }
+    }
+    void mark(int i)
+    {
+        if (c->prof_on && ev[i]) cudaEventRecord(ev[i], st);
+    }
+    void commit()
+    {
+        if (c->prof_on) c->ev_pending.push_back(ev);
+    }
+};
+
+bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const void* const* k,
+                             const void* const* v, int N, int budget, void* const* ko,
+                             void* const* vo, int32_t* idx, cudaStream_t st)
+{
+    const int pairs = R * c->layers;
+    const Shape s = shape_of(c, c->layers, R, N);
+    const int kept = budget < N ? budget : N;
+
+    QKTable tab;
+    GatherTable gt;
+    for (int i = 0; i < pairs; ++i) {
+        tab.q[i] = static_cast<const uint16_t*>(q[i]);
+        tab.k[i] = static_cast<const uint16_t*>(k[i]);
+        gt.k[i] = static_cast<const uint16_t*>(k[i]);
+        gt.v[i] = static_cast<const uint16_t*>(v[i]);
+        gt.ko[i] = static_cast<uint16_t*>(ko[i]);
+        gt.vo[i] = static_cast<uint16_t*>(vo[i]);
+    }
+    StageEvents prof(c, st);
+    const int chunks = (s.N + kChunkTokens - 1) / kChunkTokens;
+    prof.mark(0);
+    BACON_CUDA(launch_window_stats(tab, s, kChunkTokens, c->partial, st), "window_stats launch");
+    prof.mark(1);
+    BACON_CUDA(launch_window_combine(s, chunks, c->partial, c->lse2, st), "window_combine launch");
+    prof.mark(2);
+    BACON_CUDA(launch_window_scores(tab, s, c->lse2, c->B, c->Q, c->E, st), "window_scores launch");
+    prof.mark(3);
+
+    CalibArgs a;
+    a.B = c->B;
+    a.Ering = c->E;
+    a.ring = c->layers;
+    a.ring_req_stride = (long long)c->layers * c->hkv * N;
+    a.layer0 = 0;
+    a.S = c->S;
+    a.V = c->p.keep_scores ? c->V : nullptr;
+    a.Bp = c->p.keep_scores ? c->Bp : nullptr;
+    a.lambda = c->lam;
+    a.idx = idx;
+    a.budget = budget;
+    a.calib_budget = budget;
+    a.compute_scores = 1;
+    a.do_select = 1;
+    a.write_S = c->p.keep_scores;
+    a.err = c->err;
+    BACON_CUDA(launch_calibrate_select(s, calib_of(c), a, st), "calibrate_select launch");
+    prof.mark(4);
+    BACON_CUDA(launch_gather(gt, s, idx, kept, c->err, st), "gather launch");
+    prof.mark(5);
+    prof.commit();
+    c->last_units = s.units;
+    c->last_N = N;
+    return BACON_OK;
+}
+
+bacon_status check_pointer_arrays(const bacon_ctx* c, int pairs, const void* const* q,
+                                  const void* const* k, const void* const* v, void* const* ko,
+                                  void* const* vo)
+{
+    if (!q || !k || !v || !ko || !vo) return fail(BACON_EINVAL, "null pointer array");
+    for (int i = 0; i < pairs; ++i) {
+        const void* ps[] = {q[i], k[i], v[i], ko[i], vo[i]};
+        for (const void* p : ps) {
+            if (!p) return fail(BACON_EINVAL, "null tensor pointer at pair %d", i);
+            if (!aligned16(p)) return fail(BACON_EINVAL, "tensor pointer at pair %d is not 16-byte aligned", i);
+        }
+    }
+    (void)c;
+    return BACON_OK;
+}
+
+template <typename T>
+bacon_status grow(T** buf, size_t* cap, size_t bytes, const char* what)
+{
+    if (*cap >= bytes) return BACON_OK;
+    if (*buf) cudaFree(*buf);
+    *buf = nullptr;
+    *cap = 0;
+    if (cudaMalloc(reinterpret_cast<void**>(buf), bytes) != cudaSuccess) {
+        cudaGetLastError();
+        return fail(BACON_ENOMEM, "cannot allocate %zu bytes for %s", bytes, what);
+    }
+    *cap = bytes;
+    return BACON_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+void bacon_default_params(bacon_params* p)
+{
+    if (!p) return;
+    p->r = 5;
+    p->m = 4;
+    p->rho = 2;
+    p->gamma = 1.0f;
+    p->eps = 1e-8f;
+    p->use_E = 1;
+    p->use_L = 1;
+    p->use_T = 1;
+    p->keep_window = 1;
+    p->max_seq_len = 16384;
+    p->max_requests = 4;
+    p->keep_scores = 0;
+}
+
+const char* bacon_last_error(void) { return g_last_error.c_str(); }
+
+bacon_status bacon_init(bacon_ctx** out, int layers, int kv_heads, int q_heads, int head_dim,
+                        int window, int pool, int budget, const bacon_params* p)
+{
+    g_last_error.clear();
+    if (!out) return fail(BACON_EINVAL, "out is NULL");
+    *out = nullptr;
+    bacon_params prm;
+    if (p)
+        prm = *p;
+    else
+        bacon_default_params(&prm);
+    if (layers < 1 || kv_heads < 1 || q_heads < 1) return fail(BACON_EINVAL, "layers and heads must be positive");
+    if (q_heads % kv_heads) return fail(BACON_EINVAL, "q_heads %d is not a multiple of kv_heads %d", q_heads, kv_heads);
+    if (head_dim != 64 && head_dim != 128) return fail(BACON_EINVAL, "head_dim %d unsupported (64 or 128)", head_dim);
+    if (window < 1) return fail(BACON_EINVAL, "window must be positive");
+    if (pool < 1 || pool % 2 == 0) return fail(BACON_EINVAL, "pool width %d must be odd and positive", pool);
+    if (prm.r < 0 || prm.m < 0 || prm.rho < 0) return fail(BACON_EINVAL, "r, m, rho must be >= 0");
+    if (!(prm.gamma >= 0.f) || !(prm.eps >= 0.f)) return fail(BACON_EINVAL, "gamma and eps must be >= 0");
+    if (prm.max_requests < 1) return fail(BACON_EINVAL, "max_requests must be positive");
+    if ((long long)prm.max_requests * layers > kMaxPairs)
+        return fail(BACON_EINVAL, "max_requests * layers = %lld exceeds %d",
+                    (long long)prm.max_requests * layers, kMaxPairs);
+    if (prm.max_seq_len < window || prm.max_seq_len > kMaxSeq)
+        return fail(BACON_EINVAL, "max_seq_len %d outside [window, %d]", prm.max_seq_len, kMaxSeq);
+    const int group = q_heads / kv_heads;
+    const int rows = group * window;
+    if (rows > window_max_rows(head_dim))
+        return fail(BACON_EUNSUPPORTED, "group * window = %d exceeds %d for head_dim %d", rows,
+                    window_max_rows(head_dim), head_dim);
+    if (budget < 1 || (prm.keep_window && budget < window))
+        return fail(BACON_EINVAL, "budget %d invalid for window %d", budget, window);
+
+    bacon_ctx* c = new (std::nothrow) bacon_ctx();
+    if (!c) return fail(BACON_ENOMEM, "host allocation failed");
+    cudaGetDevice(&c->device);
+    c->layers = layers;
+    c->hkv = kv_heads;
+    c->hq = q_heads;
+    c->group = group;
+    c->d = head_dim;
+    c->W = window;
+    c->pool = pool;
+    c->budget = budget;
+    c->rows = rows;
+    c->p = prm;
+    c->max_chunks = (prm.max_seq_len + kChunkTokens - 1) / kChunkTokens;
+    c->unit_cap = (size_t)prm.max_requests * layers * kv_heads;
+    const size_t tok = c->unit_cap * (size_t)prm.max_seq_len;
+    cudaError_t e = cudaSuccess;
+    if (e == cudaSuccess) e = dalloc(&c->B, tok);
+    if (e == cudaSuccess) e = dalloc(&c->Q, tok);
+    if (e == cudaSuccess) e = dalloc(&c->E, tok);
+    if (e == cudaSuccess) e = dalloc(&c->S, prm.keep_scores ? tok : 0);
+    if (e == cudaSuccess) e = dalloc(&c->V, prm.keep_scores ? tok : 0);
+    if (e == cudaSuccess) e = dalloc(&c->Bp, prm.keep_scores ? tok : 0);
+    if (e == cudaSuccess) e = dalloc(&c->lam, c->unit_cap);
+    if (e == cudaSuccess) e = dalloc(&c->lse2, c->unit_cap * rows);
+    if (e == cudaSuccess) e = dalloc(&c->partial, c->unit_cap * c->max_chunks * rows);
+    if (e == cudaSuccess) e = dalloc(&c->err, 1);
+    if (e == cudaSuccess) e = cudaMemset(c->err, 0, sizeof(int));
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        free_ctx_buffers(c);
+        delete c;
+        return fail(BACON_ENOMEM, "device allocation failed: %s", cudaGetErrorString(e));
+    }
+    *out = c;
+    return BACON_OK;
+}
+
+void bacon_destroy(bacon_ctx* ctx)
+{
+    if (!ctx) return;
+    DeviceGuard dg(ctx->device);
+    cudaDeviceSynchronize();
+    free_ctx_buffers(ctx);
+    delete ctx;
+}
+
+bacon_status bacon_state_create(bacon_ctx* ctx, bacon_state** out)
+{
+    g_last_error.clear();
+    if (!ctx || !out) return fail(BACON_EINVAL, "null argument");
+    DeviceGuard dg(ctx->device);
+    bacon_state* st = new (std::nothrow) bacon_state();
+    if (!st) return fail(BACON_ENOMEM, "host allocation failed");
+    st->ctx = ctx;
+    st->ring = ctx->p.m + 1;
+    const size_t tok = (size_t)ctx->hkv * ctx->p.max_seq_len;
+    const int chunks = ctx->max_chunks;
+    cudaError_t e = dalloc(&st->Ering, tok * st->ring);
+    if (e == cudaSuccess) e = dalloc(&st->B, tok);
+    if (e == cudaSuccess) e = dalloc(&st->Q, tok);
+    if (e == cudaSuccess) e = dalloc(&st->S, tok);
+    if (e == cudaSuccess) e = dalloc(&st->lam, ctx->hkv);
+    if (e == cudaSuccess) e = dalloc(&st->lse2, (size_t)ctx->hkv * ctx->rows);
+    if (e == cudaSuccess) e = dalloc(&st->partial, (size_t)ctx->hkv * chunks * ctx->rows);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        bacon_state_destroy(st);
+        return fail(BACON_ENOMEM, "device allocation failed: %s", cudaGetErrorString(e));
+    }
+    *out = st;
+    return BACON_OK;
+}
+
+bacon_status bacon_state_reset(bacon_state* st)
+{
+    if (!st) return fail(BACON_EINVAL, "null state");
+    st->next_layer = 0;
+    st->N = 0;
+    st->scored = 0;
+    return BACON_OK;
+}
+
+void bacon_state_destroy(bacon_state* st)
+{
+    if (!st) return;
+    void* bufs[] = {st->Ering, st->B, st->Q, st->S, st->lam, st->lse2, st->partial};
+    for (void* b : bufs)
+        if (b) cudaFree(b);
+    delete st;
+}
+
+bacon_status bacon_score_layer(bacon_ctx* ctx, bacon_state* st, int layer, const void* q_win,
+                               const void* k, int seq_len, float* scores_out,
+                               bacon_stream stream)
+{
+    g_last_error.clear();
+    if (!ctx || !st || st->ctx != ctx) return fail(BACON_EINVAL, "context/state mismatch");
+    if (!q_win || !k || !aligned16(q_win) || !aligned16(k))
+        return fail(BACON_EINVAL, "q_win and k must be non-null, 16-byte aligned device pointers");
+    if (layer < 0 || layer >= ctx->layers) return fail(BACON_EINVAL, "layer %d out of range", layer);
+    if (layer != st->next_layer)
+        return fail(BACON_ESTATE, "layer %d scored out of order (expected %d)", layer, st->next_layer);
+    bacon_status rc = check_seq(ctx, seq_len, ctx->budget);
+    if (rc != BACON_OK) return rc;
+    if (layer > 0 && seq_len != st->N)
+        return fail(BACON_ESTATE, "seq_len changed within a request (%d vs %d)", seq_len, st->N);
+    DeviceGuard dg(ctx->device);
+    cudaStream_t cs = static_cast<cudaStream_t>(stream);
+
+    const Shape s = shape_of(ctx, 1, 1, seq_len);
+    QKTable tab;
+    tab.q[0] = static_cast<const uint16_t*>(q_win);
+    tab.k[0] = static_cast<const uint16_t*>(k);
+    float* Eslot = st->Ering + (size_t)(layer % st->ring) * ctx->hkv * seq_len;
+    rc = run_window(tab, s, st->partial, st->lse2, st->B, st->Q, Eslot, cs);
+    if (rc != BACON_OK) return rc;
+
+    CalibArgs a;
+    a.B = st->B;
+    a.Ering = st->Ering;
+    a.ring = st->ring;
+    a.ring_req_stride = 0;
+    a.layer0 = layer;
+    a.S = st->S;
+    a.V = nullptr;
+    a.Bp = nullptr;
+    a.lambda = st->lam;
+    a.idx = nullptr;
+    a.budget = ctx->budget;
+    a.calib_budget = ctx->budget;
+    a.compute_scores = 1;
+    a.do_select = 0;
+    a.write_S = 1;
+    a.err = ctx->err;
+    BACON_CUDA(launch_calibrate_select(s, calib_of(ctx), a, cs), "calibrate launch");
+    if (scores_out)
+        BACON_CUDA(cudaMemcpyAsync(scores_out, st->S, sizeof(float) * ctx->hkv * seq_len,
+                                   cudaMemcpyDeviceToDevice, cs),
+                   "score copy");
+    st->N = seq_len;
+    st->next_layer = layer + 1;
+    st->scored = 1;
+    return BACON_OK;
+}
+
+bacon_status bacon_select(bacon_ctx* ctx, bacon_state* st, int budget, int32_t* idx_out,
+                          bacon_stream stream)
+{
+    g_last_error.clear();
+    if (!ctx || !st || st->ctx != ctx) return fail(BACON_EINVAL, "context/state mismatch");
+    if (!st->scored) return fail(BACON_ESTATE, "no layer has been scored with this state");
+    if (!idx_out || !aligned16(idx_out)) return fail(BACON_EINVAL, "idx_out must be a 16-byte aligned device pointer");
+    bacon_status rc = check_seq(ctx, st->N, budget);
+    if (rc != BACON_OK) return rc;
+    DeviceGuard dg(ctx->device);
+    const Shape s = shape_of(ctx, 1, 1, st->N);
+    CalibArgs a;
+    a.B = st->B;
+    a.Ering = st->Ering;
+    a.ring = st->ring;
+    a.ring_req_stride = 0;
+    a.layer0 = st->next_layer - 1;
+    a.S = st->S;
+    a.V = nullptr;
+    a.Bp = nullptr;
+    a.lambda = st->lam;
+    a.idx = idx_out;
+    a.budget = budget;
+    a.calib_budget = ctx->budget;
+    a.compute_scores = 0;
+    a.do_select = 1;
+    a.write_S = 0;
+    a.err = ctx->err;
+    BACON_CUDA(launch_calibrate_select(s, calib_of(ctx), a, static_cast<cudaStream_t>(stream)),
+               "select launch");
+    return BACON_OK;
+}
+
+bacon_status bacon_compact(bacon_ctx* ctx, const void* k, const void* v, const int32_t* idx,
+                           int seq_len, int count, void* k_out, void* v_out, bacon_stream stream)
+{
+    g_last_error.clear();
+    if (!ctx) return fail(BACON_EINVAL, "null context");
+    const void* ps[] = {k, v, idx, k_out, v_out};
+    for (const void* p : ps)
+        if (!p || !aligned16(p)) return fail(BACON_EINVAL, "tensor pointers must be non-null and 16-byte aligned");
+    if (seq_len < 1 || seq_len > ctx->p.max_seq_len) return fail(BACON_EINVAL, "seq_len %d out of range", seq_len);
+    if (count < 0 || count > seq_len) return fail(BACON_EINVAL, "count %d out of range", count);
+    DeviceGuard dg(ctx->device);
+    const Shape s = shape_of(ctx, 1, 1, seq_len);
+    GatherTable gt;
+    gt.k[0] = static_cast<const uint16_t*>(k);
+    gt.v[0] = static_cast<const uint16_t*>(v);
+    gt.ko[0] = static_cast<uint16_t*>(k_out);
+    gt.vo[0] = static_cast<uint16_t*>(v_out);
+    BACON_CUDA(launch_gather(gt, s, idx, count, ctx->err, static_cast<cudaStream_t>(stream)),
+               "gather launch");
+    return BACON_OK;
+}
+
+bacon_status bacon_compress_all_layers(bacon_ctx* ctx, int requests, const void* const* q_win,
+                                       const void* const* k, const void* const* v, int seq_len,
+                                       int budget, void* const* k_out, void* const* v_out,
+                                       int32_t* idx_out, bacon_stream stream)
+{
+    g_last_error.clear();
+    if (!ctx) return fail(BACON_EINVAL, "null context");
+    if (requests < 1 || requests > ctx->p.max_requests)
+        return fail(BACON_EINVAL, "requests %d outside [1, %d]", requests, ctx->p.max_requests);
+    bacon_status rc = check_seq(ctx, seq_len, budget);
+    if (rc != BACON_OK) return rc;
+    rc = check_pointer_arrays(ctx, requests * ctx->layers, q_win, k, v, k_out, v_out);
+    if (rc != BACON_OK) return rc;
+    if (!idx_out || !aligned16(idx_out)) return fail(BACON_EINVAL, "idx_out must be a 16-byte aligned device pointer");
+    DeviceGuard dg(ctx->device);
+    return compress_device(ctx, requests, q_win, k, v, seq_len, budget, k_out, v_out, idx_out,
+                           static_cast<cudaStream_t>(stream));
+}
+
+bacon_status bacon_compress_host(bacon_ctx* ctx, int requests, const void* q_win, const void* k,
+                                 const void* v, int seq_len, int budget, void* k_out, void* v_out,
+                                 int32_t* idx_out, bacon_stream stream)
+{
+    g_last_error.clear();
+    if (!ctx) return fail(BACON_EINVAL, "null context");
+    if (!q_win || !k || !v || !k_out || !v_out || !idx_out) return fail(BACON_EINVAL, "null host buffer");
+    if (requests < 1 || requests > ctx->p.max_requests)
+        return fail(BACON_EINVAL, "requests %d outside [1, %d]", requests, ctx->p.max_requests);
+    bacon_status rc = check_seq(ctx, seq_len, budget);
+    if (rc != BACON_OK) return rc;
+    DeviceGuard dg(ctx->device);
+    cudaStream_t cs = static_cast<cudaStream_t>(stream);
+    const int pairs = requests * ctx->layers;
+    const int kept = budget < seq_len ? budget : seq_len;
+    const size_t q_pair = (size_t)ctx->hq * ctx->W * ctx->d;       // elements per (request, layer)
+    const size_t kv_pair = (size_t)ctx->hkv * seq_len * ctx->d;
+    const size_t o_pair = (size_t)ctx->hkv * kept * ctx->d;
+    const size_t idx_count = (size_t)pairs * ctx->hkv * kept;
+    if ((rc = grow(&ctx->hq_buf, &ctx->hq_cap, q_pair * pairs * 2, "queries")) != BACON_OK) return rc;
+    size_t kv_cap = ctx->hkv_cap;
+    if ((rc = grow(&ctx->hk_buf, &kv_cap, kv_pair * pairs * 2, "keys")) != BACON_OK) return rc;
+    kv_cap = ctx->hkv_cap;
+    if ((rc = grow(&ctx->hv_buf, &kv_cap, kv_pair * pairs * 2, "values")) != BACON_OK) return rc;
+    ctx->hkv_cap = kv_cap;
+    size_t o_cap = ctx->hout_cap;
+    if ((rc = grow(&ctx->hko_buf, &o_cap, o_pair * pairs * 2, "compacted keys")) != BACON_OK) return rc;
+    o_cap = ctx->hout_cap;
+    if ((rc = grow(&ctx->hvo_buf, &o_cap, o_pair * pairs * 2, "compacted values")) != BACON_OK) return rc;
+    ctx->hout_cap = o_cap;
+    if ((rc = grow(&ctx->hidx_buf, &ctx->hidx_cap, idx_count * 4, "indices")) != BACON_OK) return rc;
+
+    BACON_CUDA(cudaMemcpyAsync(ctx->hq_buf, q_win, q_pair * pairs * 2, cudaMemcpyHostToDevice, cs), "query upload");
+    BACON_CUDA(cudaMemcpyAsync(ctx->hk_buf, k, kv_pair * pairs * 2, cudaMemcpyHostToDevice, cs), "key upload");
+    BACON_CUDA(cudaMemcpyAsync(ctx->hv_buf, v, kv_pair * pairs * 2, cudaMemcpyHostToDevice, cs), "value upload");
+
+    const void* qs[kMaxPairs];
+    const void* ks[kMaxPairs];
+    const void* vs[kMaxPairs];
+    void* kos[kMaxPairs];
+    void* vos[kMaxPairs];
+    for (int i = 0; i < pairs; ++i) {
+        qs[i] = static_cast<const uint16_t*>(ctx->hq_buf) + q_pair * i;
+        ks[i] = static_cast<const uint16_t*>(ctx->hk_buf) + kv_pair * i;
+        vs[i] = static_cast<const uint16_t*>(ctx->hv_buf) + kv_pair * i;
+        kos[i] = static_cast<uint16_t*>(ctx->hko_buf) + o_pair * i;
+        vos[i] = static_cast<uint16_t*>(ctx->hvo_buf) + o_pair * i;
+    }
+    rc = compress_device(ctx, requests, qs, ks, vs, seq_len, budget, kos, vos, ctx->hidx_buf, cs);
+    if (rc != BACON_OK) return rc;
+    BACON_CUDA(cudaMemcpyAsync(k_out, ctx->hko_buf, o_pair * pairs * 2, cudaMemcpyDeviceToHost, cs), "key download");
+    BACON_CUDA(cudaMemcpyAsync(v_out, ctx->hvo_buf, o_pair * pairs * 2, cudaMemcpyDeviceToHost, cs), "value download");
+    BACON_CUDA(cudaMemcpyAsync(idx_out, ctx->hidx_buf, idx_count * 4, cudaMemcpyDeviceToHost, cs), "index download");
+    BACON_CUDA(cudaStreamSynchronize(cs), "host-path synchronisation");
+    return bacon_sync(ctx, stream);
+}
+
+bacon_status bacon_get_scores(bacon_ctx* ctx, bacon_score_kind kind, float* out, size_t count,
+                              bacon_stream stream)
+{
+    g_last_error.clear();
+    if (!ctx || !out) return fail(BACON_EINVAL, "null argument");
+    if (ctx->last_units == 0) return fail(BACON_ESTATE, "no whole-step call has run yet");
+    const size_t per_tok = (size_t)ctx->last_units * ctx->last_N;
+    const float* src = nullptr;
+    size_t n = per_tok;
+    switch (kind) {
+        case BACON_SCORE_B: src = ctx->B; break;
+        case BACON_SCORE_Q: src = ctx->Q; break;
+        case BACON_SCORE_E: src = ctx->E; break;
+        case BACON_SCORE_V: src = ctx->V; break;
+        case BACON_SCORE_BPOOL: src = ctx->Bp; break;
+        case BACON_SCORE_S: src = ctx->S; break;
+        case BACON_SCORE_LAMBDA:
+            src = ctx->lam;
+            n = ctx->last_units;
+            break;
+        default: return fail(BACON_EINVAL, "unknown score kind %d", (int)kind);
+    }
+    if (!src) return fail(BACON_ESTATE, "score kind %d is kept only with keep_scores = 1", (int)kind);
+    if (count < n) return fail(BACON_EINVAL, "output holds %zu floats, %zu needed", count, n);
+    DeviceGuard dg(ctx->device);
+    BACON_CUDA(cudaMemcpyAsync(out, src, n * sizeof(float), cudaMemcpyDeviceToDevice,
+                               static_cast<cudaStream_t>(stream)),
+               "score copy");
+    return BACON_OK;
+}
+
+bacon_status bacon_profile_enable(bacon_ctx* ctx, int enable)
+{
+    if (!ctx) return fail(BACON_EINVAL, "null context");
+    ctx->prof_on = enable ? 1 : 0;
+    return BACON_OK;
+}
+
+bacon_status bacon_profile_read(bacon_ctx* ctx, double* ms, int* launches, int n)
+{
+    if (!ctx || !ms || !launches) return fail(BACON_EINVAL, "null argument");
+    if (n < 0 || n > BACON_PROFILE_STAGES) return fail(BACON_EINVAL, "n must be in [0, %d]", BACON_PROFILE_STAGES);
+    DeviceGuard dg(ctx->device);
+    for (int i = 0; i < n; ++i) {
+        ms[i] = 0.0;
+        launches[i] = 0;
+    }
+    bacon_status rc = BACON_OK;
+    for (auto& v : ctx->ev_pending) {
+        if (v.back() && cudaEventSynchronize(v.back()) != cudaSuccess) rc = fail(BACON_ECUDA, "event wait failed");
+        for (int i = 0; i < n && rc == BACON_OK; ++i) {
+            float t = 0.f;
+            if (v[i] && v[i + 1] && cudaEventElapsedTime(&t, v[i], v[i + 1]) == cudaSuccess) {
+                ms[i] += t;
+                launches[i] += 1;
+            }
+        }
+        for (cudaEvent_t e : v)
+            if (e) ctx->ev_free.push_back(e);
+    }
+    ctx->ev_pending.clear();
+    return rc;
+}
+
+bacon_status bacon_sync(bacon_ctx* ctx, bacon_stream stream)
+{
+    if (!ctx) return fail(BACON_EINVAL, "null context");
+    DeviceGuard dg(ctx->device);
+    BACON_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)), "stream synchronisation");
+    int flag = 0;
+    BACON_CUDA(cudaMemcpy(&flag, ctx->err, sizeof(int), cudaMemcpyDeviceToHost), "error flag read");
+    if (flag) {
+        cudaMemset(ctx->err, 0, sizeof(int));
+        if (flag == 1) return fail(BACON_EINVAL, "a gather index was outside [0, seq_len)");
+        return fail(BACON_ECUDA, "device selection check failed (code %d)", flag);
+    }
+    return BACON_OK;
+}
+
+}  // extern "C"

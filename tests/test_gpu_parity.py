@@ -1,0 +1,299 @@
+"""CUDA path (through the C ABI) against the CPU oracle on the same seeded
+inputs: every configuration of the paper-shaped workloads, edge cases, the
+layer-by-layer path and the host-buffer path."""
+
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_14782_gb300 import bacon, build, workloads
+from parity import check_scores, check_selection
+
+pytestmark = pytest.mark.gpu
+
+THREADS = os.cpu_count() or 4
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    build.build()
+    bacon.load()
+
+
+def oracle_params(**kw):
+    return oracle.Params(**kw)
+
+
+def run_gpu(wl, x, budget, **kw):
+    p = bacon.default_params(keep_scores=1, max_seq_len=max(wl.seq_len, 64),
+                             max_requests=wl.requests)
+    for k, v in kw.items():
+        setattr(p, k, v)
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool,
+                        budget, params=p)
+    ko, vo, idx = ctx.compress_all_layers(x.qwin, x.k, x.v, budget)
+    ctx.sync()
+    R, Ly, H, N = wl.requests, wl.layers, wl.kv_heads, wl.seq_len
+    out = {"Kc": ko.cpu(), "Vc": vo.cpu(), "idx": idx.cpu().numpy()}
+    for kind in ("B", "Q", "E", "V", "Bpool", "S"):
+        out[kind] = ctx.scores(kind).cpu().numpy().reshape(R, Ly, H, N)
+    out["lambda"] = ctx.scores("lambda").cpu().numpy().reshape(R, Ly, H)
+    ctx.close()
+    return out
+
+
+def compare(wl, x, budget, gpu, orc, report=None):
+    """Element-wise comparison of every oracle unit; returns the swap count."""
+    N, W = wl.seq_len, wl.window
+    kb = workloads.bf16_bits(x.k)
+    vb = workloads.bf16_bits(x.v)
+    swaps = 0
+    worst = 0.0
+    kw = orc.get("_keep_window", True)
+    for key, o in orc.items():
+        if not isinstance(key, tuple):
+            continue
+        r, l, h = key
+        where = f"unit ({r},{l},{h})"
+        for name, okey in (("B", "B"), ("Q", "Q"), ("E", "E"), ("V", "V"), ("Bpool", "Bt"),
+                           ("S", "S")):
+            e, _ = check_scores(f"{where} {name}", gpu[name][r, l, h], o[okey])
+            worst = max(worst, e)
+        lam_g, lam_o = float(gpu["lambda"][r, l, h]), o["lambda"]
+        assert abs(lam_g - lam_o) <= 1e-2 * abs(lam_o) + 1e-6, (where, lam_g, lam_o)
+        gi = gpu["idx"][r, l, h]
+        swaps += check_selection(gi, o["idx"], o["S"], N, W, budget, keep_window=kw)
+        # compacted cache: bit-exact against the GPU's own indices
+        Kc = gpu["Kc"][r, l, h].view(torch.int16).numpy().view(np.uint16)
+        Vc = gpu["Vc"][r, l, h].view(torch.int16).numpy().view(np.uint16)
+        assert np.array_equal(Kc, kb[r, l, h][gi]), where
+        assert np.array_equal(Vc, vb[r, l, h][gi]), where
+    if report is not None:
+        report.update(swaps=swaps, worst_abs=worst)
+    return swaps
+
+
+def oracle_run(wl, x, budget, units=None, **kw):
+    qb = workloads.bf16_bits(x.qwin)
+    kb = workloads.bf16_bits(x.k)
+    vb = workloads.bf16_bits(x.v)
+    p = oracle_params(pool_kernel=wl.pool, **kw)
+    res = oracle.compress(qb, kb, vb, budget, p, threads=THREADS, units=units, keep_scores=True)
+    res["_keep_window"] = p.keep_window
+    return res
+
+
+# ------------------------------------------------------------ configs
+
+def test_tiny_full_parity():
+    wl = workloads.CONFIGS["tiny"]
+    x = workloads.generate(wl, seed=0, device="cuda")
+    gpu = run_gpu(wl, x, 64)
+    orc = oracle_run(wl, x, 64)
+    rep = {}
+    compare(wl, x, 64, gpu, orc, rep)
+    assert rep["swaps"] <= 2
+    # rows of the window softmax sum to one per unit
+    np.testing.assert_allclose(gpu["B"].sum(-1), 1.0, atol=1e-4)
+    np.testing.assert_allclose(gpu["Q"].sum(-1), 1.0, atol=1e-4)
+
+
+@pytest.mark.parametrize("budget", [64, 128, 256])
+def test_llava_full_parity(budget):
+    wl = workloads.CONFIGS["llava"]
+    x = workloads.generate(wl, seed=0, device="cuda")
+    gpu = run_gpu(wl, x, budget)
+    orc = oracle_run(wl, x, budget)
+    swaps = compare(wl, x, budget, gpu, orc)
+    units = wl.layers * wl.kv_heads
+    assert swaps <= max(2, units * (budget - wl.window) // 1000)
+
+
+SAMPLED = [("qwen-img", 128), ("qwen-img", 256), ("qwen-img", 512), ("video", 326),
+           ("video", 652), ("gui", 256), ("gui", 1024)]
+
+
+@pytest.mark.parametrize("name,budget", SAMPLED)
+def test_full_size_sampled_parity(name, budget):
+    """Full-size launch (as the benchmark runs it); the oracle recomputes a
+    sample of units, each with the preceding layers its persistence needs."""
+    wl = workloads.CONFIGS[name]
+    x = workloads.generate(wl, seed=0, device="cuda")
+    gpu = run_gpu(wl, x, budget)
+    R, Ly, H = wl.requests, wl.layers, wl.kv_heads
+    units = sorted({(0, 0, 0), (R - 1, Ly - 1, H - 1), (R // 2, 5, 1), (0, 4, H - 1),
+                    (R - 1, 13, 2 % H)})
+    orc = oracle_run(wl, x, budget, units=units)
+    compare(wl, x, budget, gpu, orc)
+    # whole-launch properties at every unit
+    np.testing.assert_allclose(gpu["B"].sum(-1), 1.0, atol=2e-4)
+    np.testing.assert_allclose(gpu["Q"].sum(-1), 1.0, atol=2e-4)
+    assert (gpu["E"] >= 0).all() and (gpu["V"] >= 0).all() and (gpu["lambda"] >= 0).all()
+    idx = gpu["idx"]
+    assert (np.diff(idx, axis=-1) > 0).all()
+    assert (idx[..., -wl.window:] == np.arange(wl.seq_len - wl.window, wl.seq_len)).all()
+
+
+# --------------------------------------------------------- edge cases
+
+EDGE = [
+    # name, overrides of the tiny workload, budget, oracle/GPU parameter overrides
+    ("ragged", dict(seq_len=777, visual=(16, 700)), 100, {}),
+    ("ragged_gqa_d128", dict(seq_len=1000, q_heads=6, kv_heads=2, head_dim=128,
+                             visual=(16, 900)), 96, {}),
+    ("odd_window", dict(seq_len=300, window=5, q_heads=6, kv_heads=2, visual=(16, 280)), 40, {}),
+    ("window_one", dict(seq_len=200, window=1, visual=(16, 190)), 30, {}),
+    ("no_candidates", dict(seq_len=32, visual=(0, 0), planted=0), 32, {}),
+    ("budget_is_window", dict(seq_len=400, visual=(16, 380)), 32, {}),
+    ("budget_above_n", dict(seq_len=300, visual=(16, 280)), 500, {}),
+    ("gamma_zero", dict(seq_len=640), 64, dict(gamma=0.0)),
+    ("no_window_reserve", dict(seq_len=500, visual=(16, 460)), 64, dict(keep_window=False)),
+    ("ablate_L", dict(seq_len=640, layers=6), 64, dict(use_L=False)),
+    ("ablate_E", dict(seq_len=640, layers=6), 64, dict(use_E=False)),
+    ("ablate_T", dict(seq_len=640, layers=6), 64, dict(use_T=False)),
+    ("r0_m1", dict(seq_len=640, layers=4), 64, dict(r=0, m=1)),
+    ("m0_r9", dict(seq_len=640, layers=4), 64, dict(m=0, r=9)),
+    ("m8_deep", dict(seq_len=256, layers=12, visual=(16, 200)), 48, dict(m=8)),
+    ("pool1_rho3", dict(seq_len=640), 64, dict(rho=3)),
+    ("two_requests", dict(seq_len=513, requests=2, visual=(16, 480)), 80, {}),
+    ("long_tail_chunks", dict(seq_len=3000, layers=2, visual=(16, 2900)), 200, {}),
+]
+
+
+@pytest.mark.parametrize("name,over,budget,pk", EDGE, ids=[e[0] for e in EDGE])
+def test_edge_cases(name, over, budget, pk):
+    wl = workloads.CONFIGS["tiny"].with_(**over)
+    if name == "pool1_rho3":
+        wl = wl.with_(pool=1)
+    x = workloads.generate(wl, seed=1, device="cuda")
+    gpu_kw = {k: (int(v) if isinstance(v, bool) else v) for k, v in pk.items()}
+    gpu = run_gpu(wl, x, budget, **gpu_kw)
+    orc = oracle_run(wl, x, budget, **pk)
+    compare(wl, x, budget, gpu, orc)
+    if name == "gamma_zero":
+        nc = wl.seq_len - wl.window
+        assert np.array_equal(gpu["S"][..., :nc], gpu["Bpool"][..., :nc])
+    if name == "window_one":
+        assert np.array_equal(gpu["B"], gpu["Q"]) and not gpu["E"].any()
+    if name == "budget_above_n":
+        assert (gpu["idx"] == np.arange(wl.seq_len)).all()
+
+
+# ---------------------------------------------------- planted evidence
+
+def test_planted_evidence_on_gpu():
+    from test_oracle_pins import planted_case
+    qwin, k, ev, _ = planted_case()
+    W, d = qwin.shape[1], qwin.shape[2]
+    N = k.shape[0]
+    wl = workloads.CONFIGS["tiny"].with_(layers=1, q_heads=1, kv_heads=1, head_dim=d,
+                                         seq_len=N, window=W)
+    qt = torch.tensor(qwin, dtype=torch.float32).to(torch.bfloat16).reshape(1, 1, 1, W, d)
+    kt = torch.tensor(k, dtype=torch.float32).to(torch.bfloat16).reshape(1, 1, 1, N, d)
+    x = workloads.Inputs(qt.cuda(), kt.cuda(), kt.clone().cuda(), None)
+    budget = W + 8
+    kept = {}
+    for gamma in (0.0, 1.0):
+        gpu = run_gpu(wl, x, budget, gamma=gamma)
+        orc = oracle_run(wl, x, budget, gamma=gamma)
+        compare(wl, x, budget, gpu, orc)
+        kept[gamma] = set(gpu["idx"][0, 0, 0].tolist())
+    assert not (set(ev) & kept[0.0])
+    assert set(ev) <= kept[1.0]
+
+
+# --------------------------------------------- other entry points
+
+def test_layer_path_matches_whole_step():
+    wl = workloads.CONFIGS["tiny"].with_(layers=7, q_heads=8, kv_heads=2, seq_len=900,
+                                         visual=(16, 850))
+    x = workloads.generate(wl, seed=2, device="cuda")
+    budget = 96
+    whole = run_gpu(wl, x, budget)
+    p = bacon.default_params(max_seq_len=wl.seq_len, max_requests=1)
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool,
+                        budget, params=p)
+    st = bacon.State(ctx)
+    for l in range(wl.layers):
+        S = st.score_layer(l, x.qwin[0, l], x.k[0, l], scores_out=True)
+        idx = st.select(budget, wl.seq_len)
+        ko, vo = ctx.compact(x.k[0, l], x.v[0, l], idx)
+        ctx.sync()
+        assert np.array_equal(idx.cpu().numpy(), whole["idx"][0, l]), l
+        assert np.array_equal(S.cpu().numpy(), whole["S"][0, l]), l
+        assert torch.equal(ko.cpu(), whole["Kc"][0, l]) and torch.equal(vo.cpu(), whole["Vc"][0, l])
+    # out-of-order layer and a second state's select before scoring
+    with pytest.raises(bacon.BaconError, match="ESTATE"):
+        st.score_layer(3, x.qwin[0, 3], x.k[0, 3])
+    st2 = bacon.State(ctx)
+    with pytest.raises(bacon.BaconError, match="ESTATE"):
+        st2.select(budget, wl.seq_len)
+    st2.close()
+    st.reset()
+    st.score_layer(0, x.qwin[0, 0], x.k[0, 0])
+    st.close()
+    ctx.close()
+
+
+def test_host_path_matches_device_path():
+    wl = workloads.CONFIGS["tiny"].with_(requests=2, layers=3, seq_len=700, visual=(16, 650))
+    x = workloads.generate(wl, seed=4, device="cuda")
+    budget = 80
+    dev = run_gpu(wl, x, budget)
+    p = bacon.default_params(max_seq_len=wl.seq_len, max_requests=2)
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool,
+                        budget, params=p)
+    qh, kh, vh = (t.cpu().pin_memory() for t in (x.qwin, x.k, x.v))
+    ko, vo, idx = ctx.compress_host(qh, kh, vh, budget)
+    assert np.array_equal(idx.numpy(), dev["idx"])
+    assert torch.equal(ko, dev["Kc"]) and torch.equal(vo, dev["Vc"])
+    # a second call reuses the staging buffers
+    ko2, _, idx2 = ctx.compress_host(qh, kh, vh, budget)
+    assert torch.equal(ko2, ko) and torch.equal(idx2, idx)
+    ctx.close()
+
+
+def test_out_of_range_gather_index_is_reported():
+    wl = workloads.CONFIGS["tiny"]
+    x = workloads.generate(wl, seed=0, device="cuda")
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool, 64)
+    idx = torch.zeros((wl.kv_heads, 8), dtype=torch.int32, device="cuda")
+    idx[1, 3] = wl.seq_len + 5  # checked and skipped by the kernel
+    ctx.compact(x.k[0, 0], x.v[0, 0], idx)
+    with pytest.raises(bacon.BaconError, match="gather index"):
+        ctx.sync()
+    ctx.sync()  # the flag is cleared once reported
+    ctx.close()
+
+
+def test_invalid_calls_on_gpu():
+    wl = workloads.CONFIGS["tiny"]
+    x = workloads.generate(wl, seed=0, device="cuda")
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool, 64,
+                        max_seq_len=640, max_requests=1)
+    with pytest.raises(bacon.BaconError, match="EINVAL"):
+        ctx.compress_all_layers(x.qwin, x.k, x.v, 16)  # budget below the window
+    big = workloads.CONFIGS["tiny"].with_(seq_len=700)
+    xb = workloads.generate(big, seed=0, device="cuda")
+    with pytest.raises(bacon.BaconError, match="max_seq_len"):
+        ctx.compress_all_layers(xb.qwin, xb.k, xb.v, 64)
+    with pytest.raises(bacon.BaconError, match="aligned"):
+        ctx.compact(x.k[0, 0].flatten()[1:].view(-1)[: 4 * 639 * 64].view(4, 639, 64),
+                    x.v[0, 0], torch.zeros((4, 8), dtype=torch.int32, device="cuda"))
+    ctx.close()
+
+
+def test_profile_hooks_count_launches():
+    wl = workloads.CONFIGS["tiny"]
+    x = workloads.generate(wl, seed=0, device="cuda")
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool, 64)
+    ctx.profile(True)
+    for _ in range(3):
+        ctx.compress_all_layers(x.qwin, x.k, x.v, 64)
+    prof = ctx.profile_read()
+    assert all(n == 3 for _, n in prof.values())
+    assert all(ms > 0 for ms, _ in prof.values())
+    ctx.close()
