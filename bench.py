@@ -40,6 +40,8 @@ def parse():
     ap.add_argument("--impl", choices=("bacon", "reference"), default="bacon")
     ap.add_argument("--config", default="gui")
     ap.add_argument("--budget", type=int, default=None)
+    ap.add_argument("--requests", type=int, default=None,
+                    help="override the request count (smaller profiling cases)")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -154,11 +156,14 @@ def oracle_sample(wl, budget, units, threads):
 
 def cpu_baseline(wl, budget):
     threads = min(os.cpu_count() or 1, wl.requests * wl.kv_heads)
-    units = [(r, 0, h) for r in range(wl.requests) for h in range(wl.kv_heads)]
+    layers = min(2, wl.layers)
+    units = [(r, l, h) for r in range(wl.requests) for l in range(layers)
+             for h in range(wl.kv_heads)]
     secs = oracle_sample(wl, budget, units, threads)
     return {"value": len(units) / secs, "unit": UNIT, "cores": threads, "kind": "oracle",
-            "sample": f"{len(units)} layer-heads (layer 0 of every request and kv-head) of the "
-                      f"same workload, double precision, {threads} threads, {secs:.1f} s"}
+            "sample": f"{len(units)} layer-heads (layers 0-{layers - 1} of every request and "
+                      f"kv-head) of the same workload, double precision, {threads} threads, "
+                      f"{secs:.1f} s wall"}
 
 
 def run_reference(args):
@@ -167,6 +172,8 @@ def run_reference(args):
     if rank != 0:
         return
     wl = workloads.CONFIGS[args.config]
+    if args.requests:
+        wl = wl.with_(requests=args.requests)
     budget = args.budget or max(wl.budgets)
     threads = min(os.cpu_count() or 1, wl.requests * wl.kv_heads)
     units = [(r, 0, h) for r in range(wl.requests) for h in range(wl.kv_heads)]
@@ -220,8 +227,11 @@ def main():
             dist.barrier()
 
     wl = workloads.CONFIGS[args.config]
+    if args.requests:
+        wl = wl.with_(requests=args.requests)
     budget = args.budget or max(wl.budgets)
     x = workloads.generate(wl, seed=rank, device=dev)
+    torch.cuda.empty_cache()
     p = bacon.default_params(max_seq_len=wl.seq_len, max_requests=wl.requests)
     ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool,
                         budget, params=p)
