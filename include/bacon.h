@@ -195,6 +195,33 @@ bacon_status bacon_profile_enable(bacon_ctx* ctx, int enable);
  * `n` entries; n <= BACON_PROFILE_STAGES), and clears the record. */
 bacon_status bacon_profile_read(bacon_ctx* ctx, double* ms, int* launches, int n);
 
+/* Window scores of one layer (B, Q and E of Eqs. 1, 2 and 4 for every
+ * kv-head) WITHOUT ANY DEVICE ALLOCATION.  The paper has no counterpart:
+ * this entry point exists for callers that cannot call cudaMalloc, such as
+ * a serving engine that reserves all of HBM for its KV cache up front, or
+ * code that must not pay the device-wide synchronisation of cudaMalloc /
+ * cudaFree in the middle of prefill.  It needs no context: the kernels'
+ * scratch lives in one static __device__ array of 528 KiB, which every GPU
+ * that loads the library holds until the process exits.
+ *
+ * Inputs as in the layouts above (q_win [Hq][W][d], k [Hkv][N][d] bf16);
+ * outputs B_out, Q_out, E_out fp32 [Hkv][N], all caller-owned device
+ * pointers, 16-byte aligned.  Limits: seq_len <= 16384 and
+ * q_heads * window <= 4096 (beyond them: BACON_EUNSUPPORTED); malformed
+ * arguments give BACON_EINVAL, a CUDA failure BACON_ECUDA.  No message is
+ * recorded for bacon_last_error.
+ *
+ * The first call on a device looks up the array's device address (with
+ * that device current) and caches it; make that first call before any
+ * stream capture.  Every call uses the same array: calls whose work can
+ * overlap on the GPU (different streams, or several host threads) race and
+ * must be serialised by the caller.  Nothing in the array has to start at
+ * zero: each call writes every entry it later reads. */
+bacon_status bacon_window_scores_noalloc(int kv_heads, int q_heads, int head_dim, int window,
+                                         const void* q_win, const void* k, int seq_len,
+                                         float* B_out, float* Q_out, float* E_out,
+                                         bacon_stream stream);
+
 /* Wait for the stream and report any error latched by a kernel. */
 bacon_status bacon_sync(bacon_ctx* ctx, bacon_stream stream);
 

@@ -26,7 +26,8 @@ EXPORTS = ("bacon_default_params", "bacon_init", "bacon_destroy", "bacon_last_er
            "bacon_state_create", "bacon_state_reset", "bacon_state_destroy",
            "bacon_score_layer", "bacon_select", "bacon_compact",
            "bacon_compress_all_layers", "bacon_compress_host", "bacon_get_scores",
-           "bacon_profile_enable", "bacon_profile_read", "bacon_sync")
+           "bacon_profile_enable", "bacon_profile_read", "bacon_window_scores_noalloc",
+           "bacon_sync")
 PROFILE_STAGES = ("window_stats", "window_combine", "window_scores", "calibrate_select",
                   "gather")
 
@@ -81,10 +82,13 @@ def load() -> ctypes.CDLL:
     lib.bacon_compress_host.argtypes = [_vp, _int, _vp, _vp, _vp, _int, _int, _vp, _vp, _vp, _vp]
     lib.bacon_get_scores.argtypes = [_vp, _int, _vp, ctypes.c_size_t, _vp]
     lib.bacon_sync.argtypes = [_vp, _vp]
+    lib.bacon_window_scores_noalloc.argtypes = [_int, _int, _int, _int, _vp, _vp, _int, _vp,
+                                                _vp, _vp, _vp]
     lib.bacon_profile_enable.argtypes = [_vp, _int]
     lib.bacon_profile_read.argtypes = [_vp, ctypes.POINTER(ctypes.c_double),
                                        ctypes.POINTER(_int), _int]
-    for name in ("bacon_profile_enable", "bacon_profile_read", "bacon_init", "bacon_state_create", "bacon_state_reset", "bacon_score_layer",
+    for name in ("bacon_window_scores_noalloc", "bacon_profile_enable", "bacon_profile_read",
+                 "bacon_init", "bacon_state_create", "bacon_state_reset", "bacon_score_layer",
                  "bacon_select", "bacon_compact", "bacon_compress_all_layers",
                  "bacon_compress_host", "bacon_get_scores", "bacon_sync"):
         getattr(lib, name).restype = _int

@@ -1,0 +1,92 @@
+// Window scores of one layer without any device allocation.
+//
+// Some callers cannot call cudaMalloc: a serving engine that reserves all of
+// HBM for its KV cache up front and forbids side allocations, or code that
+// must not pay the implicit device-wide synchronisation of cudaMalloc /
+// cudaFree in the middle of prefill.  For them, bacon_window_scores_noalloc
+// runs the same three window kernels as the context-based calls, but keeps
+// their scratch (pass-1 partial statistics and the per-row normalisers) in
+// one file-scope __device__ array instead of context-owned buffers.
+#include <mutex>
+
+#include "../../include/bacon.h"
+#include "common.cuh"
+
+using namespace bacon;
+
+namespace {
+
+constexpr int kMaxTotalRows = 4096;   // kv_heads * (q_heads / kv_heads) * window
+constexpr int kMaxSeq = 16384;        // tokens per call
+constexpr int kChunk = 1024;          // pass-1 token chunk, as in the context path
+constexpr int kMaxChunks = kMaxSeq / kChunk;
+constexpr int kMaxDevices = 64;
+
+// [units][chunks][rows] partial (max, sum) pairs, then [units][rows] fp32
+// normalisers packed two per float2.  528 KiB, held by every GPU that loads
+// the library until the process exits.
+static __device__ __align__(256) float2 g_scratch[kMaxTotalRows * kMaxChunks + kMaxTotalRows / 2];
+
+std::mutex g_setup_mutex;
+void* g_scratch_addr[kMaxDevices] = {};
+
+}  // namespace
+
+extern "C" {
+
+bacon_status bacon_window_scores_noalloc(int kv_heads, int q_heads, int head_dim, int window,
+                                         const void* q_win, const void* k, int seq_len,
+                                         float* B_out, float* Q_out, float* E_out,
+                                         bacon_stream stream)
+{
+    // malformed arguments
+    if (kv_heads < 1 || q_heads < 1 || q_heads % kv_heads) return BACON_EINVAL;
+    if (head_dim != 64 && head_dim != 128) return BACON_EINVAL;
+    if (window < 1 || seq_len < window) return BACON_EINVAL;
+    const void* ps[] = {q_win, k, B_out, Q_out, E_out};
+    for (const void* p : ps)
+        if (!p || (reinterpret_cast<uintptr_t>(p) & 15u)) return BACON_EINVAL;
+    // sizes beyond what the static scratch (or the kernels) can hold
+    const long long rows = (long long)(q_heads / kv_heads) * window;
+    if (seq_len > kMaxSeq || rows * kv_heads > kMaxTotalRows || rows > window_max_rows(head_dim))
+        return BACON_EUNSUPPORTED;
+
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return BACON_ECUDA;
+    float2* scratch = nullptr;
+    {
+        // one-time set-up per device, with that device current: the host-side
+        // name of the array is not a device address, so look the address up
+        std::lock_guard<std::mutex> lock(g_setup_mutex);
+        if (!g_scratch_addr[dev]) {
+            void* addr = nullptr;
+            cudaError_t e = cudaGetSymbolAddress(&addr, g_scratch);
+            if (e != cudaSuccess || !addr) return BACON_ECUDA;
+            g_scratch_addr[dev] = addr;
+        }
+        scratch = static_cast<float2*>(g_scratch_addr[dev]);
+    }
+
+    Shape s;
+    s.layers = 1;
+    s.hkv = kv_heads;
+    s.group = q_heads / kv_heads;
+    s.d = head_dim;
+    s.W = window;
+    s.N = seq_len;
+    s.units = kv_heads;
+    s.rows = (int)rows;
+    QKTable tab;
+    tab.q[0] = static_cast<const uint16_t*>(q_win);
+    tab.k[0] = static_cast<const uint16_t*>(k);
+    const int chunks = (seq_len + kChunk - 1) / kChunk;
+    float2* partial = scratch;
+    float* lse2 = reinterpret_cast<float*>(scratch + (size_t)kMaxTotalRows * kMaxChunks);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e = launch_window_stats(tab, s, kChunk, partial, st);
+    if (e == cudaSuccess) e = launch_window_combine(s, chunks, partial, lse2, st);
+    if (e == cudaSuccess) e = launch_window_scores(tab, s, lse2, B_out, Q_out, E_out, st);
+    return e == cudaSuccess ? BACON_OK : BACON_ECUDA;
+}
+
+}  // extern "C"
