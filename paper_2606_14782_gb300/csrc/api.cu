@@ -9,6 +9,7 @@
 
 #include "../../include/bacon.h"
 #include "common.cuh"
+#include "window_tc.h"
 
 using namespace bacon;
 
@@ -95,6 +96,13 @@ struct bacon_ctx {
     void* hvo_buf = nullptr;
     int32_t* hidx_buf = nullptr;
     size_t hq_cap = 0, hkv_cap = 0, hout_cap = 0, hidx_cap = 0;
+    // TMA descriptors of the last whole-step call: [kMaxPairs] K maps, then
+    // [kMaxPairs] window-query maps (device copy + pinned host staging)
+    CUtensorMap* d_maps = nullptr;
+    CUtensorMap* h_maps = nullptr;
+    cudaEvent_t maps_ev = nullptr;
+    std::vector<const void*> map_key;
+    int map_key_N = -1;
     // per-kernel timing (bacon_profile_enable)
     int prof_on = 0;
     std::vector<cudaEvent_t> ev_free;
@@ -114,6 +122,11 @@ struct bacon_state {
     float* lam = nullptr;
     float* lse2 = nullptr;
     float2* partial = nullptr;
+    CUtensorMap* d_maps = nullptr;  // [0] K map, [1] window-query map
+    CUtensorMap* h_maps = nullptr;
+    cudaEvent_t maps_ev = nullptr;
+    std::vector<const void*> map_key;
+    int map_key_N = -1;
 };
 
 namespace {
@@ -159,19 +172,64 @@ bacon_status check_seq(const bacon_ctx* c, int N, int budget)
     return BACON_OK;
 }
 
-// Eqs. 1, 2, 4 for every unit of the call: B, Q and E (E written to `E`).
-bacon_status run_window(const QKTable& tab, const Shape& s, float2* partial, float* lse2,
-                        float* B, float* Q, float* E, cudaStream_t st)
+// Encode the TMA descriptors of `pairs` (request, layer) pairs and copy them
+// to `d_maps` on the stream (K maps at [0, stride), query maps at [stride,
+// 2 stride)); skipped when the pointers and N are those of the last upload.
+bacon_status upload_maps(const bacon_ctx* c, CUtensorMap* d_maps, CUtensorMap* h_maps,
+                         cudaEvent_t ev, std::vector<const void*>& key, int& key_N, int stride,
+                         int pairs, const void* const* q, const void* const* k, int N,
+                         cudaStream_t st)
 {
-    const int chunks = (s.N + kChunkTokens - 1) / kChunkTokens;
-    BACON_CUDA(launch_window_stats(tab, s, kChunkTokens, partial, st), "window_stats launch");
-    BACON_CUDA(launch_window_combine(s, chunks, partial, lse2, st), "window_combine launch");
-    BACON_CUDA(launch_window_scores(tab, s, lse2, B, Q, E, st), "window_scores launch");
+    bool same = key_N == N && (int)key.size() == 2 * pairs;
+    for (int i = 0; same && i < pairs; ++i) same = key[2 * i] == k[i] && key[2 * i + 1] == q[i];
+    if (same) return BACON_OK;
+    BACON_CUDA(cudaEventSynchronize(ev), "descriptor staging wait");
+    for (int i = 0; i < pairs; ++i) {
+        if (!encode_rows_map(h_maps + i, k[i], c->d, (long long)c->hkv * N, kTcKBoxRows) ||
+            !encode_rows_map(h_maps + stride + i, q[i], c->d, (long long)c->hq * c->W, kTcQBoxRows))
+            return fail(BACON_ECUDA, "cuTensorMapEncodeTiled failed for pair %d", i);
+    }
+    BACON_CUDA(cudaMemcpyAsync(d_maps, h_maps, sizeof(CUtensorMap) * pairs, cudaMemcpyHostToDevice, st),
+               "descriptor upload");
+    BACON_CUDA(cudaMemcpyAsync(d_maps + stride, h_maps + stride, sizeof(CUtensorMap) * pairs,
+                               cudaMemcpyHostToDevice, st),
+               "descriptor upload");
+    BACON_CUDA(cudaEventRecord(ev, st), "descriptor event");
+    key.assign(2 * pairs, nullptr);
+    for (int i = 0; i < pairs; ++i) {
+        key[2 * i] = k[i];
+        key[2 * i + 1] = q[i];
+    }
+    key_N = N;
     return BACON_OK;
+}
+
+TcArgs tc_args(const Shape& s, const CUtensorMap* kmaps, const CUtensorMap* qmaps,
+               float2* partial, const float* lse2, float* B, float* Q, float* E, int* err)
+{
+    TcArgs a;
+    a.kmaps = kmaps;
+    a.qmaps = qmaps;
+    a.s = s;
+    a.chunks = (s.N + kTcChunkTokens - 1) / kTcChunkTokens;
+    a.total_chunks = s.units * a.chunks;
+    a.partial = partial;
+    a.lse2 = lse2;
+    a.B = B;
+    a.Q = Q;
+    a.E = E;
+    a.err = err;
+    return a;
 }
 
 void free_ctx_buffers(bacon_ctx* c)
 {
+    if (c->maps_ev) cudaEventDestroy(c->maps_ev);
+    if (c->h_maps) cudaFreeHost(c->h_maps);
+    if (c->d_maps) cudaFree(c->d_maps);
+    c->maps_ev = nullptr;
+    c->h_maps = nullptr;
+    c->d_maps = nullptr;
     for (auto& v : c->ev_pending)
         for (cudaEvent_t e : v)
             if (e) cudaEventDestroy(e);
@@ -223,24 +281,25 @@ bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const vo
     const Shape s = shape_of(c, c->layers, R, N);
     const int kept = budget < N ? budget : N;
 
-    QKTable tab;
     GatherTable gt;
     for (int i = 0; i < pairs; ++i) {
-        tab.q[i] = static_cast<const uint16_t*>(q[i]);
-        tab.k[i] = static_cast<const uint16_t*>(k[i]);
         gt.k[i] = static_cast<const uint16_t*>(k[i]);
         gt.v[i] = static_cast<const uint16_t*>(v[i]);
         gt.ko[i] = static_cast<uint16_t*>(ko[i]);
         gt.vo[i] = static_cast<uint16_t*>(vo[i]);
     }
+    bacon_status rc = upload_maps(c, c->d_maps, c->h_maps, c->maps_ev, c->map_key, c->map_key_N,
+                                  kMaxPairs, pairs, q, k, N, st);
+    if (rc != BACON_OK) return rc;
+    const TcArgs ta = tc_args(s, c->d_maps, c->d_maps + kMaxPairs, c->partial, c->lse2, c->B,
+                              c->Q, c->E, c->err);
     StageEvents prof(c, st);
-    const int chunks = (s.N + kChunkTokens - 1) / kChunkTokens;
     prof.mark(0);
-    BACON_CUDA(launch_window_stats(tab, s, kChunkTokens, c->partial, st), "window_stats launch");
+    BACON_CUDA(launch_window_stats_tc(ta, st), "window_stats launch");
     prof.mark(1);
-    BACON_CUDA(launch_window_combine(s, chunks, c->partial, c->lse2, st), "window_combine launch");
+    BACON_CUDA(launch_window_combine(s, ta.chunks, c->partial, c->lse2, st), "window_combine launch");
     prof.mark(2);
-    BACON_CUDA(launch_window_scores(tab, s, c->lse2, c->B, c->Q, c->E, st), "window_scores launch");
+    BACON_CUDA(launch_window_scores_tc(ta, st), "window_scores launch");
     prof.mark(3);
 
     CalibArgs a;
@@ -350,9 +409,8 @@ bacon_status bacon_init(bacon_ctx** out, int layers, int kv_heads, int q_heads, 
         return fail(BACON_EINVAL, "max_seq_len %d outside [window, %d]", prm.max_seq_len, kMaxSeq);
     const int group = q_heads / kv_heads;
     const int rows = group * window;
-    if (rows > window_max_rows(head_dim))
-        return fail(BACON_EUNSUPPORTED, "group * window = %d exceeds %d for head_dim %d", rows,
-                    window_max_rows(head_dim), head_dim);
+    if (rows > window_tc_max_rows())
+        return fail(BACON_EUNSUPPORTED, "group * window = %d exceeds %d", rows, window_tc_max_rows());
     if (budget < 1 || (prm.keep_window && budget < window))
         return fail(BACON_EINVAL, "budget %d invalid for window %d", budget, window);
 
@@ -384,6 +442,11 @@ bacon_status bacon_init(bacon_ctx** out, int layers, int kv_heads, int q_heads, 
     if (e == cudaSuccess) e = dalloc(&c->partial, c->unit_cap * c->max_chunks * rows);
     if (e == cudaSuccess) e = dalloc(&c->err, 1);
     if (e == cudaSuccess) e = cudaMemset(c->err, 0, sizeof(int));
+    if (e == cudaSuccess) e = dalloc(&c->d_maps, 2 * (size_t)kMaxPairs);
+    if (e == cudaSuccess)
+        e = cudaHostAlloc(reinterpret_cast<void**>(&c->h_maps), 2 * kMaxPairs * sizeof(CUtensorMap),
+                          cudaHostAllocDefault);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->maps_ev, cudaEventDisableTiming);
     if (e != cudaSuccess) {
         cudaGetLastError();
         free_ctx_buffers(c);
@@ -421,6 +484,11 @@ bacon_status bacon_state_create(bacon_ctx* ctx, bacon_state** out)
     if (e == cudaSuccess) e = dalloc(&st->lam, ctx->hkv);
     if (e == cudaSuccess) e = dalloc(&st->lse2, (size_t)ctx->hkv * ctx->rows);
     if (e == cudaSuccess) e = dalloc(&st->partial, (size_t)ctx->hkv * chunks * ctx->rows);
+    if (e == cudaSuccess) e = dalloc(&st->d_maps, 2);
+    if (e == cudaSuccess)
+        e = cudaHostAlloc(reinterpret_cast<void**>(&st->h_maps), 2 * sizeof(CUtensorMap),
+                          cudaHostAllocDefault);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&st->maps_ev, cudaEventDisableTiming);
     if (e != cudaSuccess) {
         cudaGetLastError();
         bacon_state_destroy(st);
@@ -442,9 +510,11 @@ bacon_status bacon_state_reset(bacon_state* st)
 void bacon_state_destroy(bacon_state* st)
 {
     if (!st) return;
-    void* bufs[] = {st->Ering, st->B, st->Q, st->S, st->lam, st->lse2, st->partial};
+    void* bufs[] = {st->Ering, st->B, st->Q, st->S, st->lam, st->lse2, st->partial, st->d_maps};
     for (void* b : bufs)
         if (b) cudaFree(b);
+    if (st->h_maps) cudaFreeHost(st->h_maps);
+    if (st->maps_ev) cudaEventDestroy(st->maps_ev);
     delete st;
 }
 
@@ -467,12 +537,15 @@ bacon_status bacon_score_layer(bacon_ctx* ctx, bacon_state* st, int layer, const
     cudaStream_t cs = static_cast<cudaStream_t>(stream);
 
     const Shape s = shape_of(ctx, 1, 1, seq_len);
-    QKTable tab;
-    tab.q[0] = static_cast<const uint16_t*>(q_win);
-    tab.k[0] = static_cast<const uint16_t*>(k);
     float* Eslot = st->Ering + (size_t)(layer % st->ring) * ctx->hkv * seq_len;
-    rc = run_window(tab, s, st->partial, st->lse2, st->B, st->Q, Eslot, cs);
+    rc = upload_maps(ctx, st->d_maps, st->h_maps, st->maps_ev, st->map_key, st->map_key_N, 1, 1,
+                     &q_win, &k, seq_len, cs);
     if (rc != BACON_OK) return rc;
+    const TcArgs ta = tc_args(s, st->d_maps, st->d_maps + 1, st->partial, st->lse2, st->B, st->Q,
+                              Eslot, ctx->err);
+    BACON_CUDA(launch_window_stats_tc(ta, cs), "window_stats launch");
+    BACON_CUDA(launch_window_combine(s, ta.chunks, st->partial, st->lse2, cs), "window_combine launch");
+    BACON_CUDA(launch_window_scores_tc(ta, cs), "window_scores launch");
 
     CalibArgs a;
     a.B = st->B;
@@ -707,6 +780,7 @@ bacon_status bacon_sync(bacon_ctx* ctx, bacon_stream stream)
     if (flag) {
         cudaMemset(ctx->err, 0, sizeof(int));
         if (flag == 1) return fail(BACON_EINVAL, "a gather index was outside [0, seq_len)");
+        if (flag == 3) return fail(BACON_ETIMEOUT, "a window-score kernel timed out waiting on its pipeline");
         return fail(BACON_ECUDA, "device selection check failed (code %d)", flag);
     }
     return BACON_OK;
