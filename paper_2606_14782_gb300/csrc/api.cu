@@ -7,7 +7,7 @@
 #include <string>
 #include <vector>
 
-#include "../../include/bacon.h"
+#include "bacon.h"
 #include "common.cuh"
 #include "window_tc.h"
 

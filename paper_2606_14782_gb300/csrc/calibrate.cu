@@ -30,9 +30,15 @@ __device__ SelectResult radix_select(const float* vals, int n, int k, int* hist,
     for (int shift = 24; shift >= 0; shift -= 8) {
         for (int b = threadIdx.x; b < 256; b += blockDim.x) hist[b] = 0;
         __syncthreads();
-        for (int i = threadIdx.x; i < n; i += blockDim.x) {
-            const uint32_t key = float_key(vals[i]);
-            if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1);
+        // warp-aggregated: lanes that fall into the same bin add once together
+        const int n_round = (n + 31) & ~31;
+        for (int i = threadIdx.x; i < n_round; i += blockDim.x) {
+            const bool in = i < n;
+            const uint32_t key = in ? float_key(vals[i]) : 0u;
+            const bool hit = in && (key & mask) == prefix;
+            const int bin = hit ? (int)((key >> shift) & 255u) : -1;
+            const uint32_t peers = __match_any_sync(0xffffffffu, bin);
+            if (hit && (threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
         }
         __syncthreads();
         if (threadIdx.x < 32) {
@@ -74,63 +80,123 @@ __device__ SelectResult radix_select(const float* vals, int n, int k, int* hist,
     return {prefix, remaining};
 }
 
-// Block-wide exclusive scan of one int per thread; returns the exclusive
-// prefix and writes the total to *total.
-__device__ int block_exclusive_scan(int v, int* warp_sums, int* total)
-{
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    int incl = v;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += y;
-    }
-    if (lane == 31) warp_sums[warp] = incl;
-    __syncthreads();
-    if (warp == 0) {
-        const int nw = blockDim.x >> 5;
-        int w = lane < nw ? warp_sums[lane] : 0;
-        int wi = w;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, wi, o);
-            if (lane >= o) wi += y;
-        }
-        if (lane < nw) warp_sums[lane] = wi - w;
-        if (lane == 31) *total = wi;
-    }
-    __syncthreads();
-    const int res = warp_sums[warp] + incl - v;
-    __syncthreads();
-    return res;
-}
-
-// Block-wide double sum.
-__device__ double block_sum(double v, double* red)
+// Block-wide fp32 sum by a shuffle tree (pairwise, so the rounding error
+// grows with log2 of the count).  FP64 is avoided: its rate on this part is
+// a small fraction of fp32.
+__device__ float block_sum(float v, float* red)
 {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
     if (lane == 0) red[warp] = v;
     __syncthreads();
-    double tot = 0.0;
-    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += red[w];
+    if (warp == 0) {
+        float t = lane < (int)(blockDim.x >> 5) ? red[lane] : 0.f;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        if (lane == 0) red[32] = t;
+    }
+    __syncthreads();
+    const float tot = red[32];
     __syncthreads();
     return tot;
 }
 
-// Membership in the k best of vals[0, n): key > tau, or key == tau with fewer
-// than `need` equal keys before it.  Each thread owns the contiguous index
-// range [lo, hi); `eq_before` is the number of equal keys before lo.
-struct RangeSel {
+// dst[0, n) = src[0, n) with independent 16-byte loads (n % 4 == 0 and both
+// 16-byte aligned), so the copy costs a few memory round trips, not one per
+// element.
+__device__ __forceinline__ void stage(float* dst, const float* src, int n)
+{
+    const float4* s4 = reinterpret_cast<const float4*>(src);
+    float4* d4 = reinterpret_cast<float4*>(dst);
+    const int n4 = n >> 2;
+    for (int i = threadIdx.x; i < n4; i += 4 * blockDim.x) {
+        float4 v[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+            if (i + k * (int)blockDim.x < n4) v[k] = __ldg(s4 + i + k * blockDim.x);
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+            if (i + k * (int)blockDim.x < n4) d4[i + k * blockDim.x] = v[k];
+    }
+}
+
+// Index-ordered sweeps over vals[0, n): warp w owns the contiguous segment
+// [lo, hi) and its lanes take consecutive elements, so shared-memory reads
+// are conflict-free while ballots keep the index order inside a warp.
+struct Segment {
     int lo, hi;
 };
 
-__device__ __forceinline__ RangeSel my_range(int n)
+__device__ __forceinline__ Segment warp_segment(int n)
 {
-    const int per = (n + blockDim.x - 1) / blockDim.x;
-    const int lo = min(n, (int)threadIdx.x * per);
+    const int nw = blockDim.x >> 5;
+    const int per = ((n + nw - 1) / nw + 31) & ~31;
+    const int lo = min(n, (int)(threadIdx.x >> 5) * per);
     return {lo, min(n, lo + per)};
+}
+
+__device__ __forceinline__ int warp_sum(int v)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Exclusive scan of one value per warp (lane 0's `v`), returned to every lane.
+__device__ int warp_exclusive_scan(int v, int* warp_sums, int* total)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (lane == 0) warp_sums[warp] = v;
+    __syncthreads();
+    if (warp == 0) {
+        const int nw = blockDim.x >> 5;
+        const int w = lane < nw ? warp_sums[lane] : 0;
+        int incl = w;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += y;
+        }
+        if (lane < nw) warp_sums[lane] = incl - w;
+        if (lane == 31) *total = incl;
+    }
+    __syncthreads();
+    const int r = warp_sums[warp];
+    __syncthreads();
+    return r;
+}
+
+// Walks this warp's segment in index order; calls f(i, in) for every index
+// with in = membership in the k best (key > tau, or key == tau among the
+// first `need` equal keys).  eq_before = equal keys before the segment.
+template <typename F>
+__device__ __forceinline__ void walk_topk(const float* vals, Segment sg, SelectResult sel,
+                                          int eq_before, F f)
+{
+    const int lane = threadIdx.x & 31;
+    const uint32_t lt = (1u << lane) - 1u;
+    int running = eq_before;
+    for (int base = sg.lo; base < sg.hi; base += 32) {
+        const int i = base + lane;
+        const bool valid = i < sg.hi;
+        const uint32_t key = valid ? float_key(vals[i]) : 0u;
+        const bool eq = valid && key == sel.tau;
+        const uint32_t ball = __ballot_sync(0xffffffffu, eq);
+        const int rank = running + __popc(ball & lt);
+        const bool in = valid && (key > sel.tau || (eq && rank < sel.need));
+        f(i, valid, in);
+        running += __popc(ball);
+    }
+}
+
+// Equal-to-threshold keys before this warp's segment.
+__device__ int eq_before_segment(const float* vals, Segment sg, uint32_t tau, int* warp_sums,
+                                 int* total)
+{
+    int eq = 0;
+    for (int i = sg.lo + (threadIdx.x & 31); i < sg.hi; i += 32) eq += float_key(vals[i]) == tau;
+    return warp_exclusive_scan(warp_sum(eq), warp_sums, total);
 }
 
 __global__ void __launch_bounds__(kThreads)
@@ -143,7 +209,7 @@ calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
     __shared__ int hist[256];
     __shared__ int bcast[4];
     __shared__ int warp_sums[32];
-    __shared__ double red[32];
+    __shared__ float red[33];
     __shared__ int total_s;
 
     const int u = blockIdx.x;
@@ -166,30 +232,64 @@ calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
         const int half = c.pool / 2;
         const int nprev = min(c.m, layer);
         const float inv_prev = nprev > 0 ? 1.f / (float)nprev : 0.f;
+        // B -> Vs (staging), then the pooled backbone over the candidates -> Sb
+        if ((N & 3) == 0)
+            stage(Vs, Bu, N);
+        else
+            for (int i = threadIdx.x; i < N; i += blockDim.x) Vs[i] = Bu[i];
+        __syncthreads();
         for (int i = threadIdx.x; i < N; i += blockDim.x) {
-            // pooled backbone over the candidates (positions outside ignored)
+            float mx = 0.f;
             if (i < n_cand) {
-                float mx = -INFINITY;
+                mx = -INFINITY;
                 const int lo = max(0, i - half), hi = min(n_cand - 1, i + half);
-                for (int v = lo; v <= hi; ++v) mx = fmaxf(mx, Bu[v]);
-                Sb[i] = mx;
-            } else {
-                Sb[i] = 0.f;
+                for (int v = lo; v <= hi; ++v) mx = fmaxf(mx, Vs[v]);
             }
-            // coherence: truncated radius-r box mean of E (Eqs. 5-7)
-            const int lo = max(0, i - c.r), hi = min(N - 1, i + c.r);
-            float sum = 0.f;
-            for (int v = lo; v <= hi; ++v) sum += Ec[v];
-            const float L = sum / (float)(hi - lo + 1);
-            // persistence: mean of E over the preceding min(m, l) layers (Eqs. 8-9)
-            float T = 0.f;
-            for (int j = layer - nprev; j < layer; ++j) T += Eof(j)[i];
-            T *= inv_prev;
-            float V = 0.f;
-            if (c.use_E) V += Ec[i];
-            if (c.use_L) V += L;
-            if (c.use_T) V += T;
-            Vs[i] = V;
+            Sb[i] = mx;
+        }
+        __syncthreads();
+        // E -> Vs (staging); V is built in registers, then written over it
+        if ((N & 3) == 0)
+            stage(Vs, Ec, N);
+        else
+            for (int i = threadIdx.x; i < N; i += blockDim.x) Vs[i] = Ec[i];
+        __syncthreads();
+        constexpr int kMaxPer = 24;  // N <= 24576 with 1024 threads
+        float vreg[kMaxPer];
+        // persistence: mean of E over the preceding min(m, l) layers (Eqs. 8-9)
+#pragma unroll
+        for (int k = 0; k < kMaxPer; ++k) vreg[k] = 0.f;
+        if (c.use_T) {
+            for (int j = layer - nprev; j < layer; ++j) {
+                const float* Ej = Eof(j);
+#pragma unroll
+                for (int k = 0; k < kMaxPer; ++k) {
+                    const int i = threadIdx.x + k * blockDim.x;
+                    if (i < N) vreg[k] += Ej[i];
+                }
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < kMaxPer; ++k) {
+            const int i = threadIdx.x + k * blockDim.x;
+            if (i < N) {
+                // coherence: truncated radius-r box mean of E (Eqs. 5-7)
+                const int lo = max(0, i - c.r), hi = min(N - 1, i + c.r);
+                float sum = 0.f;
+                for (int v = lo; v <= hi; ++v) sum += Vs[v];
+                const float L = sum / (float)(hi - lo + 1);
+                float V = 0.f;
+                if (c.use_E) V += Vs[i];
+                if (c.use_L) V += L;
+                if (c.use_T) V += vreg[k] * inv_prev;
+                vreg[k] = V;
+            }
+        }
+        __syncthreads();
+#pragma unroll
+        for (int k = 0; k < kMaxPer; ++k) {
+            const int i = threadIdx.x + k * blockDim.x;
+            if (i < N) Vs[i] = vreg[k];
         }
         __syncthreads();
         if (a.V) for (int i = threadIdx.x; i < N; i += blockDim.x) a.V[(size_t)u * N + i] = Vs[i];
@@ -202,42 +302,28 @@ calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
         float lam = 0.f;
         if (M > 0) {
             const SelectResult sel = radix_select(Sb, n_cand, M, hist, bcast);
-            const RangeSel rg = my_range(n_cand);
-            int eq = 0;
-            for (int i = rg.lo; i < rg.hi; ++i) eq += float_key(Sb[i]) == sel.tau;
-            int eq_before = block_exclusive_scan(eq, warp_sums, &total_s);
-            double sb = 0.0, sv = 0.0;
-            {
-                int e = eq_before;
-                for (int i = rg.lo; i < rg.hi; ++i) {
-                    const uint32_t key = float_key(Sb[i]);
-                    bool in = key > sel.tau;
-                    if (key == sel.tau) in = (e++ < sel.need);
-                    if (in) {
-                        sb += Sb[i];
-                        sv += Vs[i];
-                    }
+            const Segment sg = warp_segment(n_cand);
+            const int eqb = eq_before_segment(Sb, sg, sel.tau, warp_sums, &total_s);
+            float sb = 0.f, sv = 0.f;
+            walk_topk(Sb, sg, sel, eqb, [&](int i, bool, bool in) {
+                if (in) {
+                    sb += Sb[i];
+                    sv += Vs[i];
                 }
-            }
-            const double mb = block_sum(sb, red) / M;
-            const double mv = block_sum(sv, red) / M;
-            double vb = 0.0, vv = 0.0;
-            {
-                int e = eq_before;
-                for (int i = rg.lo; i < rg.hi; ++i) {
-                    const uint32_t key = float_key(Sb[i]);
-                    bool in = key > sel.tau;
-                    if (key == sel.tau) in = (e++ < sel.need);
-                    if (in) {
-                        const double db = Sb[i] - mb, dv = Vs[i] - mv;
-                        vb += db * db;
-                        vv += dv * dv;
-                    }
+            });
+            const float mb = block_sum(sb, red) / (float)M;
+            const float mv = block_sum(sv, red) / (float)M;
+            float vb = 0.f, vv = 0.f;  // centred second moments (two-pass)
+            walk_topk(Sb, sg, sel, eqb, [&](int i, bool, bool in) {
+                if (in) {
+                    const float db = Sb[i] - mb, dv = Vs[i] - mv;
+                    vb = fmaf(db, db, vb);
+                    vv = fmaf(dv, dv, vv);
                 }
-            }
-            const double stdb = sqrt(block_sum(vb, red) / M);
-            const double stdv = sqrt(block_sum(vv, red) / M);
-            lam = (float)((double)c.gamma * stdb / (stdv + (double)c.eps));
+            });
+            const float stdb = sqrtf(block_sum(vb, red) / (float)M);
+            const float stdv = sqrtf(block_sum(vv, red) / (float)M);
+            lam = c.gamma * stdb / (stdv + c.eps);
         }
         if (threadIdx.x == 0) a.lambda[u] = lam;
         for (int i = threadIdx.x; i < n_cand; i += blockDim.x) Sb[i] = fmaf(lam, Vs[i], Sb[i]);
@@ -255,30 +341,19 @@ calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
         for (int i = threadIdx.x; i < n_cand; i += blockDim.x) out[i] = i;
     } else if (keep > 0) {
         const SelectResult sel = radix_select(Sb, n_cand, keep, hist, bcast);
-        const RangeSel rg = my_range(n_cand);
-        int eq = 0;
-        for (int i = rg.lo; i < rg.hi; ++i) eq += float_key(Sb[i]) == sel.tau;
-        const int eq_before = block_exclusive_scan(eq, warp_sums, &total_s);
+        const Segment sg = warp_segment(n_cand);
+        const int eqb = eq_before_segment(Sb, sg, sel.tau, warp_sums, &total_s);
         int mine = 0;
-        {
-            int e = eq_before;
-            for (int i = rg.lo; i < rg.hi; ++i) {
-                const uint32_t key = float_key(Sb[i]);
-                bool in = key > sel.tau;
-                if (key == sel.tau) in = (e++ < sel.need);
-                mine += in;
-            }
-        }
-        int pos = block_exclusive_scan(mine, warp_sums, &total_s);
-        {
-            int e = eq_before;
-            for (int i = rg.lo; i < rg.hi; ++i) {
-                const uint32_t key = float_key(Sb[i]);
-                bool in = key > sel.tau;
-                if (key == sel.tau) in = (e++ < sel.need);
-                if (in) out[pos++] = i;
-            }
-        }
+        walk_topk(Sb, sg, sel, eqb, [&](int, bool, bool in) { mine += in; });
+        const int base = warp_exclusive_scan(warp_sum(mine), warp_sums, &total_s);
+        const int lane = threadIdx.x & 31;
+        const uint32_t lt = (1u << lane) - 1u;
+        int pos = base;
+        walk_topk(Sb, sg, sel, eqb, [&](int i, bool, bool in) {
+            const uint32_t ball = __ballot_sync(0xffffffffu, in);
+            if (in) out[pos + __popc(ball & lt)] = i;
+            pos += __popc(ball);
+        });
         if (threadIdx.x == 0 && total_s != keep && a.err) atomicExch(a.err, 2);
     }
     for (int w = threadIdx.x; w < win; w += blockDim.x) out[keep + w] = N - W + w;

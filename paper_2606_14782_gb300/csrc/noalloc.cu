@@ -9,7 +9,7 @@
 // one file-scope __device__ array instead of context-owned buffers.
 #include <mutex>
 
-#include "../../include/bacon.h"
+#include "bacon.h"
 #include "common.cuh"
 
 using namespace bacon;
