@@ -7,15 +7,16 @@
 //     tcgen05.mma reads directly;
 //   * one thread issues tcgen05.mma (bf16 x bf16 -> fp32) into TMEM; the
 //     accumulators never visit registers until the epilogue reads them;
-//   * eight epilogue warps (two per TMEM lane quarter, each taking half of
-//     a job's columns) turn logits into softmax statistics (pass 1) or
-//     per-token sums (pass 2) while the MMA of the next job runs into
-//     another TMEM buffer; reductions use several independent accumulators
-//     and packed fp32x2 arithmetic, exp2 runs on the SFU.
+//   * sixteen epilogue warps (four groups, each with one warp per TMEM lane
+//     quarter) share every job's columns and turn logits into softmax
+//     statistics (pass 1) or per-token sums (pass 2) while the MMA of the
+//     next job runs into another TMEM buffer; exp2 runs on the SFU.
 // Pass 1 (stats):  D[row][token], 128 rows x 128 tokens per job, 4 TMEM
-//                  buffers; a thread owns one window row and 64 tokens.
-// Pass 2 (scores): D[token][row], 128 tokens x up to 256 rows per job, 2
-//                  TMEM buffers; a thread owns one token and half the rows.
+//                  buffers; a thread owns one window row and 32 tokens.
+// Pass 2 (scores): D[token][row], 128 tokens x up to 128 rows per job, 4
+//                  TMEM buffers (so the next tile's MMA overlaps this tile's
+//                  epilogue); a thread owns one token and every fourth
+//                  16-row piece of the tile.
 // Each CTA is persistent and takes a contiguous range of 1024-token chunks
 // of the flattened (unit, chunk) space, so a CTA reloads the window rows only
 // when its range crosses into the next (request, layer, kv-head).
@@ -31,8 +32,9 @@ namespace {
 constexpr int kTileTok = 128;          // tokens per K tile
 constexpr int kChunk = 1024;           // tokens per work chunk (8 tiles)
 constexpr int kTilesPerChunk = kChunk / kTileTok;
-constexpr int kThreads = 320;          // warp 0 TMA, warp 1 MMA, warps 2-9 epilogue
-constexpr int kEpiThreads = 256;       // two epilogue warps per TMEM lane quarter
+constexpr int kGroups = 4;             // epilogue warp groups (4 warps each, one per lane quarter)
+constexpr int kEpiThreads = 128 * kGroups;
+constexpr int kThreads = 64 + kEpiThreads;  // warp 0 TMA, warp 1 MMA, then the epilogue
 constexpr int kQBox = 64;              // rows per TMA box of the window rows
 constexpr int kTmemCols = 512;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -45,7 +47,7 @@ struct Smem {
     uint32_t total;
 };
 
-template <int D>
+template <int D, int PASS>
 __host__ __device__ inline Smem smem_layout(int q_rows, int stages)
 {
     Smem s;
@@ -55,9 +57,11 @@ __host__ __device__ inline Smem smem_layout(int q_rows, int stages)
     s.q = 0;
     s.k = s.q + H * s.q_half;
     s.tables = s.k + (uint32_t)stages * s.k_stage;
-    s.xchg = s.tables + (uint32_t)q_rows * 12u;
+    // pass 2 only: per-row nl, qw and last visible key
+    s.xchg = s.tables + (PASS == 2 ? (uint32_t)q_rows * 12u : 0u);
     s.xchg = (s.xchg + 15u) & ~15u;
-    s.bars = s.xchg + 4u * 128u * 8u;  // pass 1: (m, z) per row block and row
+    // partials of groups 1.. (pass 1: per row block; pass 2: two tiles) + flags
+    s.bars = s.xchg + (kGroups - 1) * (PASS == 1 ? 4u : 2u) * 128u * 8u + 64u;
     s.bars = (s.bars + 7u) & ~7u;
     s.total = s.bars + 256u;  // barriers, TMEM base, abort flag
     return s;
@@ -119,6 +123,33 @@ __device__ inline void chunk_range(int total, int* c0, int* c1)
     *c1 = (int)(((long long)(blockIdx.x + 1) * total) / gridDim.x);
 }
 
+// Jobs of one tile.  Pass 1: n_jobs row blocks of 128 rows.  Pass 2: the
+// window rows, rounded up to 16-row granules, split into n_jobs groups of at
+// most 128 rows as evenly as granules allow.  The job loops are unrolled over
+// the four possible jobs so the sizes stay in registers.
+struct JobTable {
+    int n_jobs;
+    int n[4];
+    int row0[4];
+};
+
+__device__ __forceinline__ JobTable make_jobs(int n_jobs, int granules)
+{
+    JobTable jt;
+    jt.n_jobs = n_jobs;
+    int r = 0;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const int nj = granules == 0
+                           ? 128
+                           : 16 * (granules / n_jobs + (j < granules % n_jobs ? 1 : 0));
+        jt.n[j] = j < n_jobs ? nj : 0;
+        jt.row0[j] = r;
+        r += jt.n[j];
+    }
+    return jt;
+}
+
 // --------------------------------------------------- producer (TMA, warp 0)
 
 template <int D>
@@ -172,14 +203,14 @@ __device__ __forceinline__ void produce(const TcArgs& a, const Smem& L, uint8_t*
 // Pass 2: A = K tile (M = 128 tokens), B = window rows (N = n_h per half).
 template <int D, int PASS>
 __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* sm, const Bars& b, int stages,
-                      int q_rows, int n_jobs_per_tile, const int* job_n, const int* job_row0)
+                      int q_rows, const JobTable& jt)
 {
     const Shape& s = a.s;
     const int ntiles = (s.N + kTileTok - 1) / kTileTok;
     const uint32_t tmem = *b.tmem_base;
     const uint32_t sbase = smem_u32(sm);
-    constexpr int NBUF = PASS == 1 ? 4 : 2;
-    constexpr int BUF_COLS = PASS == 1 ? 128 : 256;
+    constexpr int NBUF = 4;
+    constexpr int BUF_COLS = 128;
     int c0, c1;
     chunk_range(a.total_chunks, &c0, &c1);
     int cur_u = -1, qwaits = 0, kt = 0, job = 0;
@@ -199,14 +230,16 @@ __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* s
             if (!tc::mbar_wait(b.k_full + st, n & 1, b.abort)) { ok = false; break; }
             tc::fence_after_sync();
             const uint32_t kaddr = sbase + L.k + st * L.k_stage;
-            for (int j = 0; j < n_jobs_per_tile; ++j, ++job) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                if (j >= jt.n_jobs) break;
                 const int buf = job % NBUF, nb = job / NBUF;
+                ++job;
                 if (!tc::mbar_wait(b.t_empty + buf, (nb & 1) ^ 1, b.abort)) { ok = false; break; }
                 tc::fence_after_sync();
                 const uint32_t d_tmem = tmem + buf * BUF_COLS;
-                const uint32_t idesc = PASS == 1 ? tc::idesc_bf16(128, 128)
-                                                 : tc::idesc_bf16(128, job_n[j]);
-                const uint32_t qaddr = sbase + L.q + job_row0[j] * 128;
+                const uint32_t idesc = tc::idesc_bf16(128, jt.n[j]);
+                const uint32_t qaddr = sbase + L.q + jt.row0[j] * 128;
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
                     const int kh = kk / 4;
@@ -233,18 +266,20 @@ __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* s
 
 // ------------------------------------------------- epilogue, pass 1 (stats)
 
-// Thread = one window row (TMEM lane) x one half (64 tokens) of every job.
+// Thread = one window row (TMEM lane) x one 32-token quarter (its group) of
+// every job; running (max, sum of 2^x) per row block, merged across the
+// groups at the end of each chunk.
 template <int D>
-__device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, uint8_t* sm, const Bars& b,
-                               int q_rows)
+__device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, uint8_t* sm,
+                                               const Bars& b, int q_rows)
 {
     const Shape& s = a.s;
     const int ntiles = (s.N + kTileTok - 1) / kTileTok;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int quarter = warp & 3;        // TMEM lanes this warp may access
-    const int half = (warp - 2) >> 2;    // which 64 tokens of each job
+    const int group = (warp - 2) >> 2;   // which 32 tokens of each job
     const uint32_t tmem = *b.tmem_base;
-    float2* xchg = reinterpret_cast<float2*>(sm + L.xchg);
+    float2* xchg = reinterpret_cast<float2*>(sm + L.xchg);  // [group - 1][rb][128]
     const int nrb = q_rows / 128;
     const float c = kLog2e * rsqrtf((float)D);
     const unsigned long long c2 = tc::pack2(c, c);
@@ -265,8 +300,8 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
         }
         const int t1 = min(ntiles, (ci + 1) * kTilesPerChunk);
         for (int t = ci * kTilesPerChunk; t < t1 && ok; ++t) {
-            const int tok0 = t * kTileTok + half * 64;
-            const bool need_mask = tok0 + 63 > s.N - s.W;
+            const int tok0 = t * kTileTok + group * 32;
+            const bool need_mask = tok0 + 31 > s.N - s.W;
 #pragma unroll
             for (int rb = 0; rb < 4; ++rb) {
                 if (rb >= nrb) break;
@@ -274,63 +309,57 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
                 ++job;
                 if (!tc::mbar_wait(b.t_full + buf, nb & 1, b.abort)) { ok = false; break; }
                 tc::fence_after_sync();
-                float v[64];
-                const uint32_t taddr =
-                    tmem + ((uint32_t)(quarter * 32) << 16) + buf * 128 + half * 64;
-                tc::tmem_ld32(taddr, v);
-                tc::tmem_ld32(taddr + 32, v + 32);
+                float v[32];
+                tc::tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + buf * 128 + group * 32, v);
                 tc::tmem_ld_wait_regs32(v);
-                tc::tmem_ld_wait_regs32(v + 32);
                 tc::fence_before_sync();
                 __syncwarp();
                 if (lane == 0) tc::mbar_arrive(b.t_empty + buf);
                 if (need_mask) {
 #pragma unroll
-                    for (int j = 0; j < 64; ++j)
+                    for (int j = 0; j < 32; ++j)
                         if (tok0 + j > vis[rb]) v[j] = -INFINITY;
                 }
-                // tree maximum of the raw logits (the scale c > 0 commutes)
-                float mx[8];
+                float mx[4];
 #pragma unroll
-                for (int i = 0; i < 8; ++i) mx[i] = tc::max3(v[8 * i], v[8 * i + 1], v[8 * i + 2]);
-#pragma unroll
-                for (int i = 0; i < 8; ++i)
-                    mx[i] = tc::max3(mx[i], v[8 * i + 3], v[8 * i + 4]);
-#pragma unroll
-                for (int i = 0; i < 8; ++i)
-                    mx[i] = tc::max3(mx[i], v[8 * i + 5], fmaxf(v[8 * i + 6], v[8 * i + 7]));
-                const float mt = tc::max3(tc::max3(mx[0], mx[1], mx[2]), tc::max3(mx[3], mx[4], mx[5]),
-                                          fmaxf(mx[6], mx[7]));
-                const float m_new = fmaxf(m_run[rb], mt * c);
+                for (int i = 0; i < 4; ++i)
+                    mx[i] = tc::max3(tc::max3(v[8 * i], v[8 * i + 1], v[8 * i + 2]),
+                                     tc::max3(v[8 * i + 3], v[8 * i + 4], v[8 * i + 5]),
+                                     fmaxf(v[8 * i + 6], v[8 * i + 7]));
+                const float m_new = fmaxf(m_run[rb], fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * c);
                 if (m_new != -INFINITY) {
                     const unsigned long long nm2 = tc::pack2(-m_new, -m_new);
-                    unsigned long long acc[4] = {0ull, 0ull, 0ull, 0ull};
+                    float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-                    for (int j = 0; j < 64; j += 2) {
+                    for (int j = 0; j < 32; j += 2) {
                         const float2 tt = tc::unpack2(tc::fma2(tc::pack2(v[j], v[j + 1]), c2, nm2));
-                        acc[(j >> 1) & 3] =
-                            tc::add2(acc[(j >> 1) & 3], tc::pack2(fast_exp2(tt.x), fast_exp2(tt.y)));
+                        acc[(j >> 1) & 3] += fast_exp2(tt.x) + fast_exp2(tt.y);
                     }
-                    const float2 s0 = tc::unpack2(tc::add2(acc[0], acc[1]));
-                    const float2 s1 = tc::unpack2(tc::add2(acc[2], acc[3]));
-                    z_run[rb] = z_run[rb] * fast_exp2(m_run[rb] - m_new) + ((s0.x + s0.y) + (s1.x + s1.y));
+                    z_run[rb] = z_run[rb] * fast_exp2(m_run[rb] - m_new) + ((acc[0] + acc[1]) + (acc[2] + acc[3]));
                     m_run[rb] = m_new;
                 }
             }
         }
         if (!ok) break;
-        // merge the two token halves of each row, then publish the chunk's partial
-        if (half == 1)
+        // merge the groups' statistics of each row, then publish the chunk's partial
+        if (group > 0)
             for (int rb = 0; rb < nrb; ++rb)
-                xchg[rb * 128 + quarter * 32 + lane] = make_float2(m_run[rb], z_run[rb]);
+                xchg[((group - 1) * 4 + rb) * 128 + quarter * 32 + lane] = make_float2(m_run[rb], z_run[rb]);
         if (!warp_barrier(b.ep_all, ep_phase, b.abort)) { ok = false; break; }
-        if (half == 0) {
+        if (group == 0) {
             for (int rb = 0; rb < nrb; ++rb) {
                 const int r = rb * 128 + quarter * 32 + lane;
-                const float2 o = xchg[rb * 128 + quarter * 32 + lane];
-                const float M = fmaxf(m_run[rb], o.x);
+                float M = m_run[rb];
+                for (int gg = 0; gg < kGroups - 1; ++gg)
+                    M = fmaxf(M, xchg[(gg * 4 + rb) * 128 + quarter * 32 + lane].x);
                 float Z = 0.f;
-                if (M != -INFINITY) Z = z_run[rb] * fast_exp2(m_run[rb] - M) + o.y * fast_exp2(o.x - M);
+                if (M != -INFINITY) {
+                    Z = z_run[rb] * fast_exp2(m_run[rb] - M);
+                    for (int gg = 0; gg < kGroups - 1; ++gg) {
+                        const float2 o = xchg[(gg * 4 + rb) * 128 + quarter * 32 + lane];
+                        Z += o.y * fast_exp2(o.x - M);
+                    }
+                }
                 if (r < s.rows)
                     a.partial[((size_t)u * a.chunks + ci) * s.rows + r] = make_float2(M, Z);
             }
@@ -350,17 +379,20 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
 // its last row is a last-position row (with W a multiple of 16 that is the
 // only place such a row can sit: FASTQ).
 struct ScoreTabs {
-    const float* nl;
-    const float* qw;
-    const int* vis;
+    const float* nl;  // [q_rows] nl, then [q_rows] qw, then [q_rows] vis
+    int q_rows;
     const uint8_t* qflag;
+    __device__ __forceinline__ const float* qw() const { return nl + q_rows; }
+    __device__ __forceinline__ const int* vis() const
+    {
+        return reinterpret_cast<const int*>(nl + 2 * q_rows);
+    }
 };
 
 template <int NV, bool FASTQ, bool MASK>
 __device__ __forceinline__ void score_chunk(const float* v, int r, const ScoreTabs& tb,
-                                            unsigned long long c2, int tok,
-                                            unsigned long long* bacc, unsigned long long* qacc,
-                                            float& qlast)
+                                            unsigned long long c2, int tok, float* bacc,
+                                            float* qacc, float& qlast)
 {
 #pragma unroll
     for (int jj = 0; jj < NV; jj += 4) {
@@ -370,19 +402,22 @@ __device__ __forceinline__ void score_chunk(const float* v, int r, const ScoreTa
         float x0 = fast_exp2(t0.x), x1 = fast_exp2(t0.y);
         float x2 = fast_exp2(t1.x), x3 = fast_exp2(t1.y);
         if (MASK) {
-            const int4 vis = *reinterpret_cast<const int4*>(tb.vis + r + jj);
+            const int4 vis = *reinterpret_cast<const int4*>(tb.vis() + r + jj);
             if (tok > vis.x) x0 = 0.f;
             if (tok > vis.y) x1 = 0.f;
             if (tok > vis.z) x2 = 0.f;
             if (tok > vis.w) x3 = 0.f;
         }
-        const unsigned long long xa = tc::pack2(x0, x1), xb = tc::pack2(x2, x3);
-        bacc[(jj >> 2) & 1] = tc::add2(bacc[(jj >> 2) & 1], xa);
-        bacc[2 + ((jj >> 2) & 1)] = tc::add2(bacc[2 + ((jj >> 2) & 1)], xb);
+        bacc[0] += x0;
+        bacc[1] += x1;
+        bacc[2] += x2;
+        bacc[3] += x3;
         if (!FASTQ) {
-            const float4 qw = *reinterpret_cast<const float4*>(tb.qw + r + jj);
-            qacc[0] = tc::fma2(xa, tc::pack2(qw.x, qw.y), qacc[0]);
-            qacc[1] = tc::fma2(xb, tc::pack2(qw.z, qw.w), qacc[1]);
+            const float4 qw = *reinterpret_cast<const float4*>(tb.qw() + r + jj);
+            qacc[0] = fmaf(x0, qw.x, qacc[0]);
+            qacc[1] = fmaf(x1, qw.y, qacc[1]);
+            qacc[0] = fmaf(x2, qw.z, qacc[0]);
+            qacc[1] = fmaf(x3, qw.w, qacc[1]);
         } else if ((jj & 15) == 12) {
             if (tb.qflag[(r + jj) >> 4]) qlast += x3;  // the group's last column
         }
@@ -390,39 +425,29 @@ __device__ __forceinline__ void score_chunk(const float* v, int r, const ScoreTa
 }
 
 template <bool FASTQ, bool MASK>
-__device__ __forceinline__ bool score_tile(int n_jobs, const int* job_n, const int* job_row0,
-                                           int& job, int half, int quarter, uint32_t tmem,
+__device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int group, int quarter,
+                                           uint32_t tmem,
                                            const Bars& b, const ScoreTabs& tb,
-                                           unsigned long long c2, int tok,
-                                           unsigned long long* bacc, unsigned long long* qacc,
-                                           float& qlast)
+                                           unsigned long long c2, int tok, float* bacc,
+                                           float* qacc, float& qlast)
 {
     const int lane = threadIdx.x & 31;
     int kglob = 0;  // 16-column piece index of the tile where this job starts
-    for (int j = 0; j < n_jobs; ++j, ++job) {
-        const int buf = job & 1, nb = job >> 1;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        if (j >= jt.n_jobs) break;
+        const int buf = job & 3, nb = job >> 2;
+        ++job;
         if (!tc::mbar_wait(b.t_full + buf, nb & 1, b.abort)) return false;
         tc::fence_after_sync();
-        const int np = job_n[j] / 16, r0 = job_row0[j];
-        const uint32_t taddr = tmem + ((uint32_t)(quarter * 32) << 16) + buf * 256;
-        // pieces i, i + 2, ... of this job; the next piece loads while this one is scored
-        int i = (half - kglob) & 1;
-        float va[16], vb[16];
-        if (i < np) {
-            tc::tmem_ld16(taddr + 16 * i, va);
-            tc::tmem_ld_wait_regs16(va);
-        }
-        while (i < np) {
-            if (i + 2 < np) tc::tmem_ld16(taddr + 16 * (i + 2), vb);
-            score_chunk<16, FASTQ, MASK>(va, r0 + 16 * i, tb, c2, tok, bacc, qacc, qlast);
-            i += 2;
-            if (i >= np) break;
-            tc::tmem_ld_wait_regs16(vb);
-            if (i + 2 < np) tc::tmem_ld16(taddr + 16 * (i + 2), va);
-            score_chunk<16, FASTQ, MASK>(vb, r0 + 16 * i, tb, c2, tok, bacc, qacc, qlast);
-            i += 2;
-            if (i >= np) break;
-            tc::tmem_ld_wait_regs16(va);
+        const int np = jt.n[j] / 16, r0 = jt.row0[j];
+        const uint32_t taddr = tmem + ((uint32_t)(quarter * 32) << 16) + buf * 128;
+        // pieces i = group, group + 4, ... of the tile that fall in this job
+        for (int i = (group - kglob) & (kGroups - 1); i < np; i += kGroups) {
+            float v[16];
+            tc::tmem_ld16(taddr + 16 * i, v);
+            tc::tmem_ld_wait_regs16(v);
+            score_chunk<16, FASTQ, MASK>(v, r0 + 16 * i, tb, c2, tok, bacc, qacc, qlast);
         }
         kglob += np;
         tc::fence_before_sync();
@@ -434,21 +459,21 @@ __device__ __forceinline__ bool score_tile(int n_jobs, const int* job_n, const i
 
 template <int D, bool FASTQ>
 __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, uint8_t* sm, const Bars& b,
-                                int q_rows, int n_jobs, const int* job_n, const int* job_row0)
+                                int q_rows, const JobTable& jt)
 {
     const Shape& s = a.s;
     const int ntiles = (s.N + kTileTok - 1) / kTileTok;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int quarter = warp & 3;
-    const int half = (warp - 2) >> 2;
-    const int et = threadIdx.x - 64;  // 0..255 among the epilogue threads
+    const int group = (warp - 2) >> 2;
+    const int et = threadIdx.x - 64;  // among the epilogue threads
     const uint32_t tmem = *b.tmem_base;
     float* nl_s = reinterpret_cast<float*>(sm + L.tables);  // [q_rows]
     float* qw_s = nl_s + q_rows;                            // [q_rows]
     int* vis_s = reinterpret_cast<int*>(qw_s + q_rows);     // [q_rows]
-    uint8_t* qflag_s = reinterpret_cast<uint8_t*>(sm + L.xchg) + 2 * 128 * 8;  // [q_rows / 16]
-    float2* xs = reinterpret_cast<float2*>(sm + L.xchg);    // [2][128]
-    const ScoreTabs tb{nl_s, qw_s, vis_s, qflag_s};
+    uint8_t* qflag_s = reinterpret_cast<uint8_t*>(sm + L.xchg) + 2 * (kGroups - 1) * 128 * 8;  // [q_rows / 16]
+    float2* xs = reinterpret_cast<float2*>(sm + L.xchg);    // [2][kGroups - 1][128]
+    const ScoreTabs tb{nl_s, q_rows, qflag_s};
     const float c = kLog2e * rsqrtf((float)D);
     const unsigned long long c2 = tc::pack2(c, c);
     int c0, c1;
@@ -475,32 +500,27 @@ __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, 
         for (int t = ci * kTilesPerChunk; t < t1 && ok; ++t) {
             const int tok = t * kTileTok + quarter * 32 + lane;
             const bool need_mask = t * kTileTok + kTileTok - 1 > s.N - s.W;
-            unsigned long long bacc[4] = {0ull, 0ull, 0ull, 0ull};
-            unsigned long long qacc[2] = {0ull, 0ull};
+            float bacc[4] = {0.f, 0.f, 0.f, 0.f};
+            float qacc[2] = {0.f, 0.f};
             float qlast = 0.f;
-            ok = need_mask ? score_tile<FASTQ, true>(n_jobs, job_n, job_row0, job, half, quarter,
-                                                     tmem, b, tb, c2, tok, bacc, qacc, qlast)
-                           : score_tile<FASTQ, false>(n_jobs, job_n, job_row0, job, half, quarter,
-                                                      tmem, b, tb, c2, tok, bacc, qacc, qlast);
+            ok = need_mask ? score_tile<FASTQ, true>(jt, job, group, quarter, tmem, b, tb, c2, tok,
+                                                     bacc, qacc, qlast)
+                           : score_tile<FASTQ, false>(jt, job, group, quarter, tmem, b, tb, c2, tok,
+                                                      bacc, qacc, qlast);
             if (!ok) break;
-            const float2 b01 = tc::unpack2(tc::add2(bacc[0], bacc[1]));
-            const float2 b23 = tc::unpack2(tc::add2(bacc[2], bacc[3]));
-            float bsum = (b01.x + b01.y) + (b23.x + b23.y);
-            float qsum;
-            if (FASTQ) {
-                qsum = qlast * (float)s.W;
-            } else {
-                const float2 qq = tc::unpack2(tc::add2(qacc[0], qacc[1]));
-                qsum = qq.x + qq.y;
-            }
-            // the two halves of a token meet in shared memory (double-buffered by tile)
-            float2* slot = xs + (t & 1) * 128 + quarter * 32 + lane;
-            if (half == 1) *slot = make_float2(bsum, qsum);
+            float bsum = (bacc[0] + bacc[1]) + (bacc[2] + bacc[3]);
+            float qsum = FASTQ ? qlast * (float)s.W : qacc[0] + qacc[1];
+            // the groups' partial sums of a token meet in shared memory
+            // (double-buffered by tile)
+            float2* slots = xs + (t & 1) * (kGroups - 1) * 128 + quarter * 32 + lane;
+            if (group > 0) slots[(group - 1) * 128] = make_float2(bsum, qsum);
             if (!warp_barrier(b.ep_pair + quarter, pair_phase, b.abort)) { ok = false; break; }
-            if (half == 0 && tok < s.N) {
-                const float2 o = *slot;
-                bsum += o.x;
-                qsum += o.y;
+            if (group == 0 && tok < s.N) {
+                for (int gg = 0; gg < kGroups - 1; ++gg) {
+                    const float2 o = slots[gg * 128];
+                    bsum += o.x;
+                    qsum += o.y;
+                }
                 const size_t idx = (size_t)u * s.N + tok;
                 a.B[idx] = bsum;
                 a.Q[idx] = qsum;
@@ -515,29 +535,15 @@ __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, 
 
 template <int D, int PASS>
 __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, int q_rows, int stages,
-                                                               int n_jobs, int n0, int n1)
+                                                               int n_jobs, int granules)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-    const Smem L = smem_layout<D>(q_rows, stages);
+    const Smem L = smem_layout<D, PASS>(q_rows, stages);
     const Bars b = bars_at(sm + L.bars, stages);
     const int warp = threadIdx.x >> 5;
-    // jobs of one tile: pass 1 = row blocks (N = 128 tokens), pass 2 = row halves
-    int job_n[4], job_row0[4];
-    if (PASS == 1) {
-        for (int j = 0; j < 4; ++j) {
-            job_n[j] = 128;
-            job_row0[j] = j * 128;
-        }
-    } else {
-        job_n[0] = n0;
-        job_row0[0] = 0;
-        job_n[1] = n1;
-        job_row0[1] = n0;
-        job_n[2] = job_n[3] = 0;
-        job_row0[2] = job_row0[3] = 0;
-    }
+    const JobTable jt = make_jobs(n_jobs, granules);
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < stages; ++i) {
@@ -552,7 +558,7 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, int q_
         tc::mbar_init(b.q_empty, 1);
         tc::mbar_init(b.drain, 1);
         tc::mbar_init(b.ep_all, kEpiThreads / 32);
-        for (int i = 0; i < 4; ++i) tc::mbar_init(b.ep_pair + i, 2);
+        for (int i = 0; i < 4; ++i) tc::mbar_init(b.ep_pair + i, kGroups);
         *b.abort = 0;
         tc::fence_barrier_init();
     }
@@ -567,15 +573,14 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, int q_
     if (warp == 0) {
         if (tc::elect_one()) produce<D>(a, L, sm, b, stages, q_rows);
     } else if (warp == 1) {
-        if (tc::elect_one())
-            issue<D, PASS>(a, L, sm, b, stages, q_rows, n_jobs, job_n, job_row0);
+        if (tc::elect_one()) issue<D, PASS>(a, L, sm, b, stages, q_rows, jt);
     } else {
         if (PASS == 1)
             epilogue_stats<D>(a, L, sm, b, q_rows);
         else if (a.s.W % 16 == 0)
-            epilogue_scores<D, true>(a, L, sm, b, q_rows, n_jobs, job_n, job_row0);
+            epilogue_scores<D, true>(a, L, sm, b, q_rows, jt);
         else
-            epilogue_scores<D, false>(a, L, sm, b, q_rows, n_jobs, job_n, job_row0);
+            epilogue_scores<D, false>(a, L, sm, b, q_rows, jt);
     }
 
     tc::fence_before_sync();
@@ -607,24 +612,12 @@ cudaError_t launch_impl(const TcArgs& a, cudaStream_t st)
     const int rows = a.s.rows;
     // pass 1: whole 128-row MMA blocks; pass 2: whole 64-row TMA boxes
     const int q_rows = PASS == 1 ? (rows + 127) / 128 * 128 : (rows + kQBox - 1) / kQBox * kQBox;
-    int n0 = 0, n1 = 0, n_jobs = 1;
-    if (PASS == 1) {
-        n_jobs = q_rows / 128;
-    } else {
-        const int r16 = (rows + 15) / 16 * 16;
-        if (r16 <= 256) {
-            n0 = r16;
-            n_jobs = 1;
-        } else {
-            n0 = (r16 / 2 + 15) / 16 * 16;
-            n1 = r16 - n0;
-            n_jobs = 2;
-        }
-    }
+    const int granules = PASS == 1 ? 0 : (rows + 15) / 16;
+    const int n_jobs = PASS == 1 ? q_rows / 128 : (granules + 7) / 8;
     int stages = 4;
     const size_t budget = 227 * 1024 - 1024;
-    while (stages > 2 && smem_layout<D>(q_rows, stages).total > budget) --stages;
-    const Smem L = smem_layout<D>(q_rows, stages);
+    while (stages > 2 && smem_layout<D, PASS>(q_rows, stages).total > budget) --stages;
+    const Smem L = smem_layout<D, PASS>(q_rows, stages);
     if (L.total > budget) return cudaErrorInvalidValue;
     // at least half of the SM's shared memory: one CTA (and one 512-column
     // TMEM allocation) per SM
@@ -634,7 +627,7 @@ cudaError_t launch_impl(const TcArgs& a, cudaStream_t st)
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
     if (e != cudaSuccess) return e;
     const int grid = a.total_chunks < num_sms() ? a.total_chunks : num_sms();
-    window_tc_kernel<D, PASS><<<grid, kThreads, bytes, st>>>(a, q_rows, stages, n_jobs, n0, n1);
+    window_tc_kernel<D, PASS><<<grid, kThreads, bytes, st>>>(a, q_rows, stages, n_jobs, granules);
     return cudaGetLastError();
 }
 
