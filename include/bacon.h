@@ -201,13 +201,15 @@ bacon_status bacon_profile_read(bacon_ctx* ctx, double* ms, int* launches, int n
  * a serving engine that reserves all of HBM for its KV cache up front, or
  * code that must not pay the device-wide synchronisation of cudaMalloc /
  * cudaFree in the middle of prefill.  It needs no context: the kernels'
- * scratch lives in one static __device__ array of 528 KiB, which every GPU
- * that loads the library holds until the process exits.
+ * scratch (softmax statistics and two TMA descriptors) lives in one static
+ * __device__ array of about 528 KiB, which every GPU that loads the library
+ * holds until the process exits.
  *
  * Inputs as in the layouts above (q_win [Hq][W][d], k [Hkv][N][d] bf16);
  * outputs B_out, Q_out, E_out fp32 [Hkv][N], all caller-owned device
- * pointers, 16-byte aligned.  Limits: seq_len <= 16384 and
- * q_heads * window <= 4096 (beyond them: BACON_EUNSUPPORTED); malformed
+ * pointers, 16-byte aligned.  Limits: seq_len <= 16384,
+ * q_heads * window <= 4096 and (q_heads / kv_heads) * window <= 512 (beyond
+ * them: BACON_EUNSUPPORTED); malformed
  * arguments give BACON_EINVAL, a CUDA failure BACON_ECUDA.  No message is
  * recorded for bacon_last_error.
  *

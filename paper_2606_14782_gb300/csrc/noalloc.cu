@@ -5,12 +5,15 @@
 // must not pay the implicit device-wide synchronisation of cudaMalloc /
 // cudaFree in the middle of prefill.  For them, bacon_window_scores_noalloc
 // runs the same three window kernels as the context-based calls, but keeps
-// their scratch (pass-1 partial statistics and the per-row normalisers) in
-// one file-scope __device__ array instead of context-owned buffers.
+// their scratch (pass-1 partial statistics, the per-row normalisers and the
+// two TMA descriptors) in one file-scope __device__ array instead of
+// context-owned buffers.
+#include <cstring>
 #include <mutex>
 
 #include "bacon.h"
 #include "common.cuh"
+#include "window_tc.h"
 
 using namespace bacon;
 
@@ -22,10 +25,14 @@ constexpr int kChunk = 1024;          // pass-1 token chunk, as in the context p
 constexpr int kMaxChunks = kMaxSeq / kChunk;
 constexpr int kMaxDevices = 64;
 
+constexpr int kMapBytes = 2 * sizeof(CUtensorMap);  // K map, window-query map
+
 // [units][chunks][rows] partial (max, sum) pairs, then [units][rows] fp32
-// normalisers packed two per float2.  528 KiB, held by every GPU that loads
-// the library until the process exits.
-static __device__ __align__(256) float2 g_scratch[kMaxTotalRows * kMaxChunks + kMaxTotalRows / 2];
+// normalisers packed two per float2, then the two 128-byte TMA descriptors.
+// 528.25 KiB, held by every GPU that loads the library until the process
+// exits.
+static __device__ __align__(256) float2
+    g_scratch[kMaxTotalRows * kMaxChunks + kMaxTotalRows / 2 + kMapBytes / sizeof(float2)];
 
 std::mutex g_setup_mutex;
 void* g_scratch_addr[kMaxDevices] = {};
@@ -48,7 +55,7 @@ bacon_status bacon_window_scores_noalloc(int kv_heads, int q_heads, int head_dim
         if (!p || (reinterpret_cast<uintptr_t>(p) & 15u)) return BACON_EINVAL;
     // sizes beyond what the static scratch (or the kernels) can hold
     const long long rows = (long long)(q_heads / kv_heads) * window;
-    if (seq_len > kMaxSeq || rows * kv_heads > kMaxTotalRows || rows > window_max_rows(head_dim))
+    if (seq_len > kMaxSeq || rows * kv_heads > kMaxTotalRows || rows > window_tc_max_rows())
         return BACON_EUNSUPPORTED;
 
     int dev = 0;
@@ -76,16 +83,35 @@ bacon_status bacon_window_scores_noalloc(int kv_heads, int q_heads, int head_dim
     s.N = seq_len;
     s.units = kv_heads;
     s.rows = (int)rows;
-    QKTable tab;
-    tab.q[0] = static_cast<const uint16_t*>(q_win);
-    tab.k[0] = static_cast<const uint16_t*>(k);
     const int chunks = (seq_len + kChunk - 1) / kChunk;
     float2* partial = scratch;
     float* lse2 = reinterpret_cast<float*>(scratch + (size_t)kMaxTotalRows * kMaxChunks);
+    CUtensorMap* maps =
+        reinterpret_cast<CUtensorMap*>(scratch + (size_t)kMaxTotalRows * kMaxChunks + kMaxTotalRows / 2);
+    // descriptors are encoded on the host and copied from this stack buffer;
+    // a copy from pageable memory is staged before cudaMemcpyAsync returns
+    alignas(64) CUtensorMap host_maps[2];
+    if (!encode_rows_map(&host_maps[0], k, head_dim, (long long)kv_heads * seq_len, kTcKBoxRows) ||
+        !encode_rows_map(&host_maps[1], q_win, head_dim, (long long)q_heads * window, kTcQBoxRows))
+        return BACON_ECUDA;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    cudaError_t e = launch_window_stats(tab, s, kChunk, partial, st);
+    if (cudaMemcpyAsync(maps, host_maps, sizeof host_maps, cudaMemcpyHostToDevice, st) != cudaSuccess)
+        return BACON_ECUDA;
+    TcArgs a;
+    a.kmaps = maps;
+    a.qmaps = maps + 1;
+    a.s = s;
+    a.chunks = chunks;
+    a.total_chunks = s.units * chunks;
+    a.partial = partial;
+    a.lse2 = lse2;
+    a.B = B_out;
+    a.Q = Q_out;
+    a.E = E_out;
+    a.err = nullptr;
+    cudaError_t e = launch_window_stats_tc(a, st);
     if (e == cudaSuccess) e = launch_window_combine(s, chunks, partial, lse2, st);
-    if (e == cudaSuccess) e = launch_window_scores(tab, s, lse2, B_out, Q_out, E_out, st);
+    if (e == cudaSuccess) e = launch_window_scores_tc(a, st);
     return e == cudaSuccess ? BACON_OK : BACON_ECUDA;
 }
 

@@ -531,6 +531,28 @@ __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, 
     if (!ok) raise_abort(b, a.err);
 }
 
+// ------------------------------------------------------------------ merge
+
+// Per (unit, window row): log2 of the softmax normaliser over all chunks,
+// plus log2(G W), so that pass 2's 2^(logit' - lse2) is A_{q,i} / (G W).
+__global__ void window_combine_kernel(Shape s, int chunks, const float2* __restrict__ partial,
+                                      float* __restrict__ lse2)
+{
+    const int u = blockIdx.x;
+    const float log2_gw = log2f((float)s.rows);
+    for (int r = threadIdx.x; r < s.rows; r += blockDim.x) {
+        const float2* p = partial + (size_t)u * chunks * s.rows + r;
+        float M = -INFINITY;
+        for (int c = 0; c < chunks; ++c) M = fmaxf(M, p[(size_t)c * s.rows].x);
+        float Z = 0.f;
+        for (int c = 0; c < chunks; ++c) {
+            const float2 v = p[(size_t)c * s.rows];
+            if (v.y > 0.f) Z += v.y * exp2f(v.x - M);
+        }
+        lse2[(size_t)u * s.rows + r] = M + log2f(Z) + log2_gw;
+    }
+}
+
 // --------------------------------------------------------------- kernels
 
 template <int D, int PASS>
@@ -634,6 +656,15 @@ cudaError_t launch_impl(const TcArgs& a, cudaStream_t st)
 }  // namespace
 
 int window_tc_max_rows() { return 512; }
+
+cudaError_t launch_window_combine(const Shape& s, int chunks, const float2* partial,
+                                  float* lse2, cudaStream_t st)
+{
+    const int threads = s.rows < 512 ? ((s.rows + 31) / 32) * 32 : 512;
+    window_combine_kernel<<<s.units, threads, 0, st>>>(s, chunks, partial, lse2);
+    return cudaGetLastError();
+}
+
 
 cudaError_t launch_window_stats_tc(const TcArgs& a, cudaStream_t st)
 {

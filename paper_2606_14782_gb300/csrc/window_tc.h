@@ -28,10 +28,11 @@ constexpr int kTcChunkTokens = 1024;
 // Largest G * W the tcgen05 kernels take.
 int window_tc_max_rows();
 
-// Pass 1 / pass 2 on the tensor cores; the merge between them is
-// launch_window_combine.
+// Pass 1 / pass 2 on the tensor cores, and the merge between them.
 cudaError_t launch_window_stats_tc(const TcArgs& a, cudaStream_t st);
 cudaError_t launch_window_scores_tc(const TcArgs& a, cudaStream_t st);
+cudaError_t launch_window_combine(const Shape& s, int chunks, const float2* partial, float* lse2,
+                                  cudaStream_t st);
 
 // 2-D tensor map over `rows` rows of d bf16 values at `base`: boxes of
 // 64 columns x box_rows rows, 128-byte swizzle, zero fill out of bounds.
