@@ -205,6 +205,22 @@ def run_reference(args):
 
 # ------------------------------------------------------------ GPU arm
 
+def reduce_step_time(ms: float, world: int, device) -> float:
+    """Replicas run independently; the job is as slow as its slowest rank."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(units_per_rank: int, world: int, ms: float) -> float:
+    """Whole-job layer-heads per second: every rank's units over the slowest time."""
+    return world * units_per_rank / (ms / 1e3)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -266,14 +282,10 @@ def main():
     prof = ctx.profile_read()
     ctx.profile(False)
     ctx.sync()
-    ms = e0.elapsed_time(e1) / args.steps
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = reduce_step_time(e0.elapsed_time(e1) / args.steps, world, dev)
 
     units = wl.requests * wl.layers * wl.kv_heads
-    value = world * units / (ms / 1e3)
+    value = job_throughput(units, world, ms)
     hbm, tflops, tflops_sus, peak_src = peaks()
 
     # per-kernel times measured live (CUDA events around each launch)
@@ -344,14 +356,10 @@ def main():
             ctx.compress_host(hq, hk, hv, budget, hko, hvo, hidx)
         f1.record(stream)
         torch.cuda.synchronize()
-        e2e_ms = f0.elapsed_time(f1) / args.e2e_steps
-        if world > 1:
-            t = torch.tensor([e2e_ms], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_ms = float(t.item())
+        e2e_ms = reduce_step_time(f0.elapsed_time(f1) / args.e2e_steps, world, dev)
         h2d = sum(t.numel() * t.element_size() for t in (hq, hk, hv))
         d2h = sum(t.numel() * t.element_size() for t in (hko, hvo, hidx))
-        line["e2e"] = {"value": world * units / (e2e_ms / 1e3), "unit": UNIT,
+        line["e2e"] = {"value": job_throughput(units, world, e2e_ms), "unit": UNIT,
                        "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d,
                        "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
                        "path": "bacon_compress_host (pinned host buffers)"}
