@@ -150,6 +150,30 @@ bacon_status bacon_compress_all_layers(bacon_ctx* ctx, int requests,
                                        void* const* v_out, int32_t* idx_out,
                                        bacon_stream stream);
 
+/* The whole step with one budget per layer (window included), e.g. the
+ * pyramid schedule of bacon_pyramid_budgets (PyramidKV-style allocation,
+ * Sec. 5 / App. B: BACON replaces only the within-head score, the base
+ * compressor's layer budgets are kept).  layer_budgets is a HOST array of
+ * `layers` ints; K_{l,h} of Eq. 12 is the layer's own budget minus W.
+ * idx_out is a HOST array of DEVICE pointers [request * layers + layer], each
+ * int32 [Hkv][kept_l] with kept_l = min(layer_budgets[l], seq_len); k_out and
+ * v_out point at [Hkv][kept_l][d] per pair.  Other arguments and errors as
+ * bacon_compress_all_layers. */
+bacon_status bacon_compress_layer_budgets(bacon_ctx* ctx, int requests,
+                                          const void* const* q_win, const void* const* k,
+                                          const void* const* v, int seq_len,
+                                          const int* layer_budgets, void* const* k_out,
+                                          void* const* v_out, int32_t* const* idx_out,
+                                          bacon_stream stream);
+
+/* Pyramid budget schedule over `layers` layers averaging `budget` (window
+ * included): with K = budget - window, K_min = floor(K / beta) and
+ * K_max = 2 K - K_min, layer l keeps W + K_min +
+ * floor((layers - 1 - l) (K_max - K_min) / (layers - 1)) tokens, so the first
+ * layer keeps the most, the last the fewest, and the layers together keep
+ * at most layers x budget.  Host-only; writes out[0 .. layers). */
+void bacon_pyramid_budgets(int layers, int window, int budget, int beta, int* out);
+
 /* The same step on HOST buffers: inputs are copied to library-owned device
  * buffers, compressed, and the outputs copied back, all on `stream`; the
  * call returns once the outputs are on the host.  Contiguous host layouts:

@@ -112,6 +112,7 @@ def _lib_handle():
             lib.bo_select.restype = c_int
             lib.bo_gather.argtypes = [_U16, c_int, c_int, _I32, c_int, _U16]
             lib.bo_bf16_to_double.argtypes = [_U16, ctypes.c_long, _D]
+            lib.bo_pyramid_budgets.argtypes = [c_int, c_int, c_int, c_int, _I32]
             _lib = lib
     return _lib
 
@@ -241,6 +242,14 @@ def select(S, N, W, budget, params: Params):
     return idx[:n].copy(), gap.value
 
 
+def pyramid_budgets(layers, window, budget, beta=20):
+    """Per-layer budgets of the PyramidKV-style schedule (window included)."""
+    out = np.empty(max(1, layers), dtype=np.int32)
+    _lib_handle().bo_pyramid_budgets(int(layers), int(window), int(budget), int(beta),
+                                     _p(out, _I32))
+    return out[:layers].copy()
+
+
 def gather(x_bits, idx):
     """Compacted cache rows x[idx] (bf16 bit patterns, bitwise copy)."""
     x = np.ascontiguousarray(x_bits, dtype=np.uint16)
@@ -269,10 +278,14 @@ def compress(qwin_bits, k_bits, v_bits, budget, params: Params | None = None,
     of (request, layer, kv_head); the residuals of the preceding layers that
     the persistence term needs are then computed as well.
 
+    ``budget`` is one budget for every layer or a sequence of per-layer
+    budgets (window included).
+
     Returns a dict keyed by (r, l, h) with 'idx', 'gap', 'lambda', 'Kc', 'Vc'
     and, when keep_scores, the score arrays of ``score_unit``.
     """
     params = params or Params()
+    layer_budget = (lambda l: int(budget[l])) if hasattr(budget, "__len__") else (lambda l: int(budget))
     R, Ly, Hq, W, d = qwin_bits.shape
     _, _, Hkv, N, _ = k_bits.shape
     G = Hq // Hkv
@@ -298,9 +311,9 @@ def compress(qwin_bits, k_bits, v_bits, budget, params: Params | None = None,
                 E_of[l] = residual(Q, B)
                 continue
             prev = [E_of[j] for j in persistence_layers(l, params.m)]
-            sc = score_unit(q, kk, prev, params, budget)
+            sc = score_unit(q, kk, prev, params, layer_budget(l))
             E_of[l] = sc["E"]
-            idx, gap = select(sc["S"], N, W, budget, params)
+            idx, gap = select(sc["S"], N, W, layer_budget(l), params)
             entry = {"idx": idx, "gap": gap, "lambda": sc["lambda"],
                      "Kc": gather(k_bits[r, l, h], idx),
                      "Vc": gather(v_bits[r, l, h], idx)}

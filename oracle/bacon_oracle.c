@@ -315,3 +315,21 @@ void bo_gather(const uint16_t* x, int N, int d, const int32_t* idx,
         memcpy(out + (size_t)j * d, x + (size_t)idx[j] * d,
                sizeof(uint16_t) * (size_t)d);
 }
+
+/* Layer budgets of a linear pyramid from K_max at the first layer to K_min
+ * at the last, each rounded down so that the total never exceeds the
+ * uniform candidate budget K per layer. */
+void bo_pyramid_budgets(int layers, int window, int budget, int beta, int* out)
+{
+    const int K = budget - window;
+    if (layers <= 1) {
+        if (layers == 1) out[0] = budget;
+        return;
+    }
+    const int K_min = K / beta;
+    const int K_max = 2 * K - K_min;
+    for (int l = 0; l < layers; ++l) {
+        const long long rise = (long long)(layers - 1 - l) * (K_max - K_min) / (layers - 1);
+        out[l] = K_min + (int)rise + window;
+    }
+}

@@ -94,6 +94,14 @@ int bo_score_unit(const double* qwin, const double* k, int G, int W, int N,
 int bo_select(const double* S, int N, int W, int budget, const bo_params* p,
               int32_t* idx, double* gap);
 
+/* PyramidKV-style layer budgets (a base-compressor schedule BACON plugs into,
+ * Sec. 5 / App. B): with K = budget - W candidates kept per layer on
+ * average, K_min = floor(K / beta), K_max = 2 K - K_min, layer l keeps
+ * K_min + floor((layers - 1 - l) (K_max - K_min) / (layers - 1)) candidates
+ * (K for a single layer), plus the W window tokens.  out[l] = that budget;
+ * the layers together keep at most layers x K candidates. */
+void bo_pyramid_budgets(int layers, int window, int budget, int beta, int* out);
+
 /* Compacted cache: out[j] = x[idx[j]] row-wise, d values per row, bitwise. */
 void bo_gather(const uint16_t* x, int N, int d, const int32_t* idx,
                int count, uint16_t* out);

@@ -27,7 +27,7 @@ EXPORTS = ("bacon_default_params", "bacon_init", "bacon_destroy", "bacon_last_er
            "bacon_score_layer", "bacon_select", "bacon_compact",
            "bacon_compress_all_layers", "bacon_compress_host", "bacon_get_scores",
            "bacon_profile_enable", "bacon_profile_read", "bacon_window_scores_noalloc",
-           "bacon_sync")
+           "bacon_compress_layer_budgets", "bacon_pyramid_budgets", "bacon_sync")
 PROFILE_STAGES = ("window_stats", "window_combine", "window_scores", "calibrate_select",
                   "gather")
 
@@ -82,12 +82,19 @@ def load() -> ctypes.CDLL:
     lib.bacon_compress_host.argtypes = [_vp, _int, _vp, _vp, _vp, _int, _int, _vp, _vp, _vp, _vp]
     lib.bacon_get_scores.argtypes = [_vp, _int, _vp, ctypes.c_size_t, _vp]
     lib.bacon_sync.argtypes = [_vp, _vp]
+    lib.bacon_compress_layer_budgets.argtypes = [_vp, _int, ctypes.POINTER(_vp),
+                                                 ctypes.POINTER(_vp), ctypes.POINTER(_vp), _int,
+                                                 ctypes.POINTER(_int), ctypes.POINTER(_vp),
+                                                 ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp]
+    lib.bacon_pyramid_budgets.argtypes = [_int, _int, _int, _int, ctypes.POINTER(_int)]
+    lib.bacon_pyramid_budgets.restype = None
     lib.bacon_window_scores_noalloc.argtypes = [_int, _int, _int, _int, _vp, _vp, _int, _vp,
                                                 _vp, _vp, _vp]
     lib.bacon_profile_enable.argtypes = [_vp, _int]
     lib.bacon_profile_read.argtypes = [_vp, ctypes.POINTER(ctypes.c_double),
                                        ctypes.POINTER(_int), _int]
-    for name in ("bacon_window_scores_noalloc", "bacon_profile_enable", "bacon_profile_read",
+    for name in ("bacon_compress_layer_budgets", "bacon_window_scores_noalloc",
+                 "bacon_profile_enable", "bacon_profile_read",
                  "bacon_init", "bacon_state_create", "bacon_state_reset", "bacon_score_layer",
                  "bacon_select", "bacon_compact", "bacon_compress_all_layers",
                  "bacon_compress_host", "bacon_get_scores", "bacon_sync"):
@@ -192,6 +199,31 @@ class Context:
         self._last_units, self._last_N = R * Ly * self.kv_heads, N
         return k_out, v_out, idx_out
 
+    def compress_layer_budgets(self, qwin, k, v, layer_budgets, stream=None):
+        """Per-layer budgets (window included).  Returns lists indexed
+        [request][layer] of k_out [Hkv, kept_l, d], v_out and idx [Hkv, kept_l]."""
+        R, Ly, Hq, W, d = qwin.shape
+        N = k.shape[3]
+        assert len(layer_budgets) == Ly
+        kept = [min(int(b), N) for b in layer_budgets]
+        ko = [[torch.empty((self.kv_heads, kept[l], d), dtype=k.dtype, device=k.device)
+               for l in range(Ly)] for _ in range(R)]
+        vo = [[torch.empty_like(ko[r][l]) for l in range(Ly)] for r in range(R)]
+        ix = [[torch.empty((self.kv_heads, kept[l]), dtype=torch.int32, device=k.device)
+               for l in range(Ly)] for _ in range(R)]
+        pairs = [(r, l) for r in range(R) for l in range(Ly)]
+        tq = _ptr_array([qwin[r, l].data_ptr() for r, l in pairs])
+        tk = _ptr_array([k[r, l].data_ptr() for r, l in pairs])
+        tv = _ptr_array([v[r, l].data_ptr() for r, l in pairs])
+        tko = _ptr_array([ko[r][l].data_ptr() for r, l in pairs])
+        tvo = _ptr_array([vo[r][l].data_ptr() for r, l in pairs])
+        tix = _ptr_array([ix[r][l].data_ptr() for r, l in pairs])
+        b = (_int * Ly)(*[int(x) for x in layer_budgets])
+        _check(load().bacon_compress_layer_budgets(self.handle, R, tq, tk, tv, N, b, tko, tvo,
+                                                   tix, _stream_ptr(stream)))
+        self._last_units, self._last_N = R * Ly * self.kv_heads, N
+        return ko, vo, ix
+
     def compress_host(self, qwin, k, v, budget, k_out=None, v_out=None, idx_out=None,
                       stream=None):
         """The same step on host (CPU, ideally pinned) tensors; blocks until
@@ -253,6 +285,13 @@ class Context:
                                     count, k_out.data_ptr(), v_out.data_ptr(),
                                     _stream_ptr(stream)))
         return k_out, v_out
+
+
+def pyramid_budgets(layers, window, budget, beta=20):
+    """The library's pyramid budget schedule (bacon_pyramid_budgets)."""
+    out = (_int * layers)()
+    load().bacon_pyramid_budgets(layers, window, budget, beta, out)
+    return list(out)
 
 
 class State:

@@ -273,20 +273,29 @@ struct StageEvents {
     }
 };
 
+// The whole step.  layer_budget[l] is the budget of layer l (window
+// included); idx[pair] receives the pair's [Hkv][min(budget, N)] positions.
 bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const void* const* k,
-                             const void* const* v, int N, int budget, void* const* ko,
-                             void* const* vo, int32_t* idx, cudaStream_t st)
+                             const void* const* v, int N, const int* layer_budget,
+                             void* const* ko, void* const* vo, int32_t* const* idx,
+                             cudaStream_t st)
 {
     const int pairs = R * c->layers;
     const Shape s = shape_of(c, c->layers, R, N);
-    const int kept = budget < N ? budget : N;
 
     GatherTable gt;
+    CalibArgs a;
     for (int i = 0; i < pairs; ++i) {
+        const int budget = layer_budget[i % c->layers];
         gt.k[i] = static_cast<const uint16_t*>(k[i]);
         gt.v[i] = static_cast<const uint16_t*>(v[i]);
         gt.ko[i] = static_cast<uint16_t*>(ko[i]);
         gt.vo[i] = static_cast<uint16_t*>(vo[i]);
+        gt.idx[i] = idx[i];
+        gt.kept[i] = budget < N ? budget : N;
+        a.idx[i] = idx[i];
+        a.budget[i] = budget;
+        a.calib_budget[i] = budget;
     }
     bacon_status rc = upload_maps(c, c->d_maps, c->h_maps, c->maps_ev, c->map_key, c->map_key_N,
                                   kMaxPairs, pairs, q, k, N, st);
@@ -302,7 +311,6 @@ bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const vo
     BACON_CUDA(launch_window_scores_tc(ta, st), "window_scores launch");
     prof.mark(3);
 
-    CalibArgs a;
     a.B = c->B;
     a.Ering = c->E;
     a.ring = c->layers;
@@ -312,16 +320,13 @@ bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const vo
     a.V = c->p.keep_scores ? c->V : nullptr;
     a.Bp = c->p.keep_scores ? c->Bp : nullptr;
     a.lambda = c->lam;
-    a.idx = idx;
-    a.budget = budget;
-    a.calib_budget = budget;
     a.compute_scores = 1;
     a.do_select = 1;
     a.write_S = c->p.keep_scores;
     a.err = c->err;
     BACON_CUDA(launch_calibrate_select(s, calib_of(c), a, st), "calibrate_select launch");
     prof.mark(4);
-    BACON_CUDA(launch_gather(gt, s, idx, kept, c->err, st), "gather launch");
+    BACON_CUDA(launch_gather(gt, s, c->err, st), "gather launch");
     prof.mark(5);
     prof.commit();
     c->last_units = s.units;
@@ -557,9 +562,9 @@ bacon_status bacon_score_layer(bacon_ctx* ctx, bacon_state* st, int layer, const
     a.V = nullptr;
     a.Bp = nullptr;
     a.lambda = st->lam;
-    a.idx = nullptr;
-    a.budget = ctx->budget;
-    a.calib_budget = ctx->budget;
+    a.idx[0] = nullptr;
+    a.budget[0] = ctx->budget;
+    a.calib_budget[0] = ctx->budget;
     a.compute_scores = 1;
     a.do_select = 0;
     a.write_S = 1;
@@ -596,9 +601,9 @@ bacon_status bacon_select(bacon_ctx* ctx, bacon_state* st, int budget, int32_t* 
     a.V = nullptr;
     a.Bp = nullptr;
     a.lambda = st->lam;
-    a.idx = idx_out;
-    a.budget = budget;
-    a.calib_budget = ctx->budget;
+    a.idx[0] = idx_out;
+    a.budget[0] = budget;
+    a.calib_budget[0] = ctx->budget;
     a.compute_scores = 0;
     a.do_select = 1;
     a.write_S = 0;
@@ -625,8 +630,9 @@ bacon_status bacon_compact(bacon_ctx* ctx, const void* k, const void* v, const i
     gt.v[0] = static_cast<const uint16_t*>(v);
     gt.ko[0] = static_cast<uint16_t*>(k_out);
     gt.vo[0] = static_cast<uint16_t*>(v_out);
-    BACON_CUDA(launch_gather(gt, s, idx, count, ctx->err, static_cast<cudaStream_t>(stream)),
-               "gather launch");
+    gt.idx[0] = idx;
+    gt.kept[0] = count;
+    BACON_CUDA(launch_gather(gt, s, ctx->err, static_cast<cudaStream_t>(stream)), "gather launch");
     return BACON_OK;
 }
 
@@ -645,8 +651,50 @@ bacon_status bacon_compress_all_layers(bacon_ctx* ctx, int requests, const void*
     if (rc != BACON_OK) return rc;
     if (!idx_out || !aligned16(idx_out)) return fail(BACON_EINVAL, "idx_out must be a 16-byte aligned device pointer");
     DeviceGuard dg(ctx->device);
-    return compress_device(ctx, requests, q_win, k, v, seq_len, budget, k_out, v_out, idx_out,
-                           static_cast<cudaStream_t>(stream));
+    const int kept = budget < seq_len ? budget : seq_len;
+    std::vector<int> budgets(ctx->layers, budget);
+    int32_t* idx_pairs[kMaxPairs];
+    for (int i = 0; i < requests * ctx->layers; ++i) idx_pairs[i] = idx_out + (size_t)i * ctx->hkv * kept;
+    return compress_device(ctx, requests, q_win, k, v, seq_len, budgets.data(), k_out, v_out,
+                           idx_pairs, static_cast<cudaStream_t>(stream));
+}
+
+bacon_status bacon_compress_layer_budgets(bacon_ctx* ctx, int requests, const void* const* q_win,
+                                          const void* const* k, const void* const* v,
+                                          int seq_len, const int* layer_budgets,
+                                          void* const* k_out, void* const* v_out,
+                                          int32_t* const* idx_out, bacon_stream stream)
+{
+    g_last_error.clear();
+    if (!ctx) return fail(BACON_EINVAL, "null context");
+    if (requests < 1 || requests > ctx->p.max_requests)
+        return fail(BACON_EINVAL, "requests %d outside [1, %d]", requests, ctx->p.max_requests);
+    if (!layer_budgets || !idx_out) return fail(BACON_EINVAL, "null budget or index array");
+    for (int l = 0; l < ctx->layers; ++l) {
+        bacon_status rc = check_seq(ctx, seq_len, layer_budgets[l]);
+        if (rc != BACON_OK) return rc;
+    }
+    bacon_status rc = check_pointer_arrays(ctx, requests * ctx->layers, q_win, k, v, k_out, v_out);
+    if (rc != BACON_OK) return rc;
+    for (int i = 0; i < requests * ctx->layers; ++i)
+        if (!idx_out[i] || !aligned16(idx_out[i]))
+            return fail(BACON_EINVAL, "index pointer of pair %d must be a 16-byte aligned device pointer", i);
+    DeviceGuard dg(ctx->device);
+    return compress_device(ctx, requests, q_win, k, v, seq_len, layer_budgets, k_out, v_out,
+                           idx_out, static_cast<cudaStream_t>(stream));
+}
+
+void bacon_pyramid_budgets(int layers, int window, int budget, int beta, int* out)
+{
+    if (!out || layers < 1) return;
+    const int K = budget - window;
+    if (layers == 1 || beta < 1 || K <= 0) {
+        for (int l = 0; l < layers; ++l) out[l] = budget;
+        return;
+    }
+    const int lo = K / beta, hi = 2 * K - lo;
+    for (int l = 0; l < layers; ++l)
+        out[l] = window + lo + (int)((long long)(layers - 1 - l) * (hi - lo) / (layers - 1));
 }
 
 bacon_status bacon_compress_host(bacon_ctx* ctx, int requests, const void* q_win, const void* k,
@@ -697,7 +745,10 @@ bacon_status bacon_compress_host(bacon_ctx* ctx, int requests, const void* q_win
         kos[i] = static_cast<uint16_t*>(ctx->hko_buf) + o_pair * i;
         vos[i] = static_cast<uint16_t*>(ctx->hvo_buf) + o_pair * i;
     }
-    rc = compress_device(ctx, requests, qs, ks, vs, seq_len, budget, kos, vos, ctx->hidx_buf, cs);
+    std::vector<int> budgets(ctx->layers, budget);
+    int32_t* idx_pairs[kMaxPairs];
+    for (int i = 0; i < pairs; ++i) idx_pairs[i] = ctx->hidx_buf + (size_t)i * ctx->hkv * kept;
+    rc = compress_device(ctx, requests, qs, ks, vs, seq_len, budgets.data(), kos, vos, idx_pairs, cs);
     if (rc != BACON_OK) return rc;
     BACON_CUDA(cudaMemcpyAsync(k_out, ctx->hko_buf, o_pair * pairs * 2, cudaMemcpyDeviceToHost, cs), "key download");
     BACON_CUDA(cudaMemcpyAsync(v_out, ctx->hvo_buf, o_pair * pairs * 2, cudaMemcpyDeviceToHost, cs), "value download");

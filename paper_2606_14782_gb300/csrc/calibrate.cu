@@ -218,7 +218,7 @@ calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
     const int layer = a.layer0 + (pair - rq * s.layers);
     const int win = c.keep_window ? W : 0;
     const int n_cand = N - win;
-    const int kept_total = min(a.budget, N);
+    const int kept_total = min(a.budget[pair], N);
     const int keep = kept_total - win;
 
     auto Eof = [&](int j) -> const float* {
@@ -296,7 +296,7 @@ calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
         if (a.Bp) for (int i = threadIdx.x; i < N; i += blockDim.x) a.Bp[(size_t)u * N + i] = Sb[i];
 
         // Eqs. 12-15
-        const int calib_keep = min(a.calib_budget, N) - win;
+        const int calib_keep = min(a.calib_budget[pair], N) - win;
         const long long Ml = (long long)c.rho * (long long)(calib_keep > 0 ? calib_keep : 0);
         const int M = (int)(Ml < n_cand ? Ml : n_cand);
         float lam = 0.f;
@@ -336,7 +336,7 @@ calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
     }
 
     if (!a.do_select) return;
-    int32_t* out = a.idx + (size_t)u * kept_total;
+    int32_t* out = a.idx[pair] + (size_t)h * kept_total;
     if (keep >= n_cand) {
         for (int i = threadIdx.x; i < n_cand; i += blockDim.x) out[i] = i;
     } else if (keep > 0) {

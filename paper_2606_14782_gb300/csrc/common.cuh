@@ -15,6 +15,8 @@ struct GatherTable {
     const uint16_t* v[kMaxPairs];
     uint16_t* ko[kMaxPairs];
     uint16_t* vo[kMaxPairs];
+    const int32_t* idx[kMaxPairs];  // [Hkv][kept] kept positions of the pair
+    int kept[kMaxPairs];             // rows kept per kv-head
 };
 
 // Geometry of one call.  A "unit" is one (request, layer, kv-head); units
@@ -76,9 +78,9 @@ struct CalibArgs {
     float* V;            // optional [units][N]
     float* Bp;           // optional [units][N]
     float* lambda;       // [units]
-    int32_t* idx;        // [units][kept] (written when do_select)
-    int budget;          // kept tokens per head (window included)
-    int calib_budget;    // budget that sets K in Eq. 12
+    int32_t* idx[kMaxPairs];     // per (request, layer): [Hkv][kept] (written when do_select)
+    int budget[kMaxPairs];       // kept tokens per head (window included)
+    int calib_budget[kMaxPairs]; // budget that sets K in Eq. 12
     int compute_scores;  // 1: V, B~, lambda, S from B and the residuals
     int do_select;       // 1: top-B selection into idx
     int write_S;
@@ -90,8 +92,7 @@ cudaError_t launch_calibrate_select(const Shape& s, const Calib& c, const CalibA
 // Dynamic shared memory of the calibration kernel for N tokens.
 size_t calibrate_smem(int N);
 
-// Gather of the kept K/V rows.
-cudaError_t launch_gather(const GatherTable& tab, const Shape& s, const int32_t* idx, int kept,
-                          int* err, cudaStream_t st);
+// Gather of the kept K/V rows (kept counts may differ between pairs).
+cudaError_t launch_gather(const GatherTable& tab, const Shape& s, int* err, cudaStream_t st);
 
 }  // namespace bacon

@@ -9,16 +9,16 @@ namespace bacon {
 namespace {
 
 __global__ void __launch_bounds__(256)
-gather_kernel(GatherTable tab, Shape s, const int32_t* __restrict__ idx, int kept,
-              int* __restrict__ err)
+gather_kernel(GatherTable tab, Shape s, int* __restrict__ err)
 {
     const int u = blockIdx.y;
     const int pair = u / s.hkv, h = u - pair * s.hkv;
+    const int kept = tab.kept[pair];
     const int cpr = s.d / 8;
     const int e = blockIdx.x * blockDim.x + threadIdx.x;
     const int j = e / cpr, q = e - j * cpr;
     if (j >= kept) return;
-    const int src = idx[(size_t)u * kept + j];
+    const int src = tab.idx[pair][(size_t)h * kept + j];
     if (src < 0 || src >= s.N) {
         if (err) atomicExch(err, 1);
         return;
@@ -37,13 +37,14 @@ gather_kernel(GatherTable tab, Shape s, const int32_t* __restrict__ idx, int kep
 
 }  // namespace
 
-cudaError_t launch_gather(const GatherTable& tab, const Shape& s, const int32_t* idx, int kept,
-                          int* err, cudaStream_t st)
+cudaError_t launch_gather(const GatherTable& tab, const Shape& s, int* err, cudaStream_t st)
 {
+    int kept = 0;
+    for (int p = 0; p < s.units / s.hkv; ++p) kept = tab.kept[p] > kept ? tab.kept[p] : kept;
     if (kept <= 0) return cudaSuccess;
     const int pieces = kept * (s.d / 8);
     dim3 grid((pieces + 255) / 256, s.units);
-    gather_kernel<<<grid, 256, 0, st>>>(tab, s, idx, kept, err);
+    gather_kernel<<<grid, 256, 0, st>>>(tab, s, err);
     return cudaGetLastError();
 }
 

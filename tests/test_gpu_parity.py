@@ -297,3 +297,63 @@ def test_profile_hooks_count_launches():
     assert all(n == 3 for _, n in prof.values())
     assert all(ms > 0 for ms, _ in prof.values())
     ctx.close()
+
+
+# ------------------------------------------------ per-layer budgets (PyramidKV)
+
+def _compare_layer_budgets(wl, x, budgets, ko, vo, ix, orc):
+    N, W = wl.seq_len, wl.window
+    kb = workloads.bf16_bits(x.k)
+    vb = workloads.bf16_bits(x.v)
+    swaps = 0
+    for key, o in orc.items():
+        if not isinstance(key, tuple):
+            continue
+        r, l, h = key
+        gi = ix[r][l][h].cpu().numpy()
+        swaps += check_selection(gi, o["idx"], o["S"], N, W, int(budgets[l]))
+        Kc = ko[r][l][h].cpu().view(torch.int16).numpy().view(np.uint16)
+        Vc = vo[r][l][h].cpu().view(torch.int16).numpy().view(np.uint16)
+        assert np.array_equal(Kc, kb[r, l, h][gi]) and np.array_equal(Vc, vb[r, l, h][gi])
+    return swaps
+
+
+@pytest.mark.parametrize("name,budget,beta", [("tiny", 64, 4), ("llava", 128, 20),
+                                              ("qwen-img", 256, 20)])
+def test_pyramid_layer_budgets_parity(name, budget, beta):
+    wl = workloads.CONFIGS[name].with_(layers=min(8, workloads.CONFIGS[name].layers))
+    x = workloads.generate(wl, seed=3, device="cuda")
+    budgets = bacon.pyramid_budgets(wl.layers, wl.window, budget, beta)
+    assert budgets == oracle.pyramid_budgets(wl.layers, wl.window, budget, beta).tolist()
+    p = bacon.default_params(keep_scores=1, max_seq_len=wl.seq_len, max_requests=wl.requests)
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool,
+                        budget, params=p)
+    ko, vo, ix = ctx.compress_layer_budgets(x.qwin, x.k, x.v, budgets)
+    ctx.sync()
+    S = ctx.scores("S").cpu().numpy().reshape(wl.requests, wl.layers, wl.kv_heads, wl.seq_len)
+    ctx.close()
+    units = None if name == "tiny" else [(0, l, h) for l in (0, 3, wl.layers - 1)
+                                           for h in (0, wl.kv_heads - 1)]
+    orc = oracle_run(wl, x, budgets, units=units)
+    for key, o in orc.items():
+        if isinstance(key, tuple):
+            check_scores(f"S {key}", S[key], o["S"])
+    _compare_layer_budgets(wl, x, budgets, ko, vo, ix, orc)
+    # the first layer keeps the most tokens, the last the fewest
+    assert ix[0][0].shape[1] >= ix[0][-1].shape[1]
+
+
+def test_uniform_layer_budgets_match_whole_step():
+    wl = workloads.CONFIGS["tiny"].with_(layers=4, requests=2, seq_len=700, visual=(16, 650))
+    x = workloads.generate(wl, seed=6, device="cuda")
+    whole = run_gpu(wl, x, 96)
+    p = bacon.default_params(max_seq_len=wl.seq_len, max_requests=2)
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool, 96,
+                        params=p)
+    ko, vo, ix = ctx.compress_layer_budgets(x.qwin, x.k, x.v, [96] * wl.layers)
+    ctx.sync()
+    for r in range(2):
+        for l in range(wl.layers):
+            assert np.array_equal(ix[r][l].cpu().numpy(), whole["idx"][r, l])
+            assert torch.equal(ko[r][l].cpu(), whole["Kc"][r, l])
+    ctx.close()

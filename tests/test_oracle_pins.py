@@ -472,3 +472,41 @@ def test_compress_driver_threads_and_subsets():
     want = oracle.score_unit(q, kk, Es[3:5], p, 64)
     got = oracle.compress(qb, kb, vb, 64, p, units=[(0, 5, 1)], keep_scores=True)[(0, 5, 1)]
     assert np.array_equal(got["T"], want["T"]) and got["lambda"] == want["lambda"]
+
+
+# ------------------------------------------------ PyramidKV layer budgets
+
+def test_pyramid_budgets_hand_worked():
+    # K = 10 candidates per layer on average, beta 5: K_min = 2, K_max = 18,
+    # three layers -> 18, 10, 2 (+ window 4)
+    assert oracle.pyramid_budgets(3, 4, 14, 5).tolist() == [22, 14, 6]
+    # a single layer keeps the uniform budget
+    assert oracle.pyramid_budgets(1, 8, 64, 20).tolist() == [64]
+
+
+@pytest.mark.parametrize("layers,window,budget,beta", [(28, 64, 1024, 20), (32, 32, 64, 20),
+                                                     (28, 32, 256, 5), (7, 16, 100, 3)])
+def test_pyramid_budgets_properties(layers, window, budget, beta):
+    b = oracle.pyramid_budgets(layers, window, budget, beta)
+    K = budget - window
+    assert b[0] - window == 2 * K - K // beta
+    assert b[-1] - window == K // beta
+    assert all(x >= y for x, y in zip(b, b[1:]))          # pyramid: never grows with depth
+    assert all(x >= window for x in b)
+    # the schedule spends the uniform budget, never more (floor per layer)
+    assert layers * K - (layers - 1) <= int((b - window).sum()) <= layers * K
+
+
+def test_compress_accepts_layer_budgets():
+    from paper_2606_14782_gb300 import workloads
+    wl = workloads.CONFIGS["tiny"].with_(layers=3, seq_len=300, visual=(16, 280))
+    x = workloads.generate(wl, seed=2)
+    qb, kb, vb = (workloads.bf16_bits(t) for t in (x.qwin, x.k, x.v))
+    budgets = oracle.pyramid_budgets(3, wl.window, 64, 4)
+    res = oracle.compress(qb, kb, vb, budgets, oracle.Params(), threads=2)
+    for (r, l, h), o in res.items():
+        assert o["idx"].size == budgets[l]
+        # each layer matches a uniform run at that layer's budget
+    one = oracle.compress(qb, kb, vb, int(budgets[1]), oracle.Params(), threads=2,
+                          units=[(0, 1, 2)])
+    assert np.array_equal(one[(0, 1, 2)]["idx"], res[(0, 1, 2)]["idx"])
