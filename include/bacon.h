@@ -166,6 +166,26 @@ bacon_status bacon_compress_layer_budgets(bacon_ctx* ctx, int requests,
                                           void* const* v_out, int32_t* const* idx_out,
                                           bacon_stream stream);
 
+/* The whole step with AdaKV-style adaptive head budgets (Sec. 5 / App. B:
+ * the base compressor spreads a layer's budget over its kv-heads; BACON
+ * supplies the score, Eq. 16, with K of Eq. 12 the average per-head budget).
+ * Per (request, layer), with K = min(budget, N) - W per head on average:
+ * every head first keeps its own top floor(alpha K) candidates; the other
+ * Hkv K - Hkv floor(alpha K) slots go to the best remaining candidates of
+ * all heads together (larger score first, ties to the lower head, then the
+ * lower position).  Outputs are flat per (request, layer) pair, heads in
+ * order: idx_out[pair] -> int32 [Hkv * kept] (each head's kept positions
+ * ascending, then its window), k_out/v_out[pair] -> [Hkv * kept][d], with
+ * kept = min(budget, N); counts_out is a DEVICE int32 [requests][layers][Hkv]
+ * array receiving each head's kept count (window included).  alpha in
+ * [0, 1]; BACON_EUNSUPPORTED when kv_heads x candidates exceeds 204800.
+ * Other arguments and errors as bacon_compress_all_layers. */
+bacon_status bacon_compress_adaptive(bacon_ctx* ctx, int requests, const void* const* q_win,
+                                     const void* const* k, const void* const* v, int seq_len,
+                                     int budget, float alpha, void* const* k_out,
+                                     void* const* v_out, int32_t* const* idx_out,
+                                     int32_t* counts_out, bacon_stream stream);
+
 /* Pyramid budget schedule over `layers` layers averaging `budget` (window
  * included): with K = budget - window, K_min = floor(K / beta) and
  * K_max = 2 K - K_min, layer l keeps W + K_min +

@@ -113,6 +113,9 @@ def _lib_handle():
             lib.bo_gather.argtypes = [_U16, c_int, c_int, _I32, c_int, _U16]
             lib.bo_bf16_to_double.argtypes = [_U16, ctypes.c_long, _D]
             lib.bo_pyramid_budgets.argtypes = [c_int, c_int, c_int, c_int, _I32]
+            lib.bo_select_adaptive.argtypes = [_D, c_int, c_int, c_int, c_int, c_double,
+                                               ctypes.POINTER(_Params), _I32, _I32]
+            lib.bo_select_adaptive.restype = c_int
             _lib = lib
     return _lib
 
@@ -250,6 +253,21 @@ def pyramid_budgets(layers, window, budget, beta=20):
     return out[:layers].copy()
 
 
+def select_adaptive(S_heads, W, budget, alpha, params: Params):
+    """AdaKV-style selection over the heads of one (request, layer).
+    S_heads [H, N].  Returns a list of per-head ascending kept positions."""
+    S = _f64(S_heads)
+    H, N = S.shape
+    idx = np.empty((H, N), dtype=np.int32)
+    counts = np.empty(H, dtype=np.int32)
+    cp = params._c()
+    rc = _lib_handle().bo_select_adaptive(_p(S), H, N, int(W), int(budget), float(alpha),
+                                          ctypes.byref(cp), _p(idx, _I32), _p(counts, _I32))
+    if rc != 0:
+        raise ValueError("oracle: invalid adaptive selection arguments")
+    return [idx[h, :counts[h]].copy() for h in range(H)]
+
+
 def gather(x_bits, idx):
     """Compacted cache rows x[idx] (bf16 bit patterns, bitwise copy)."""
     x = np.ascontiguousarray(x_bits, dtype=np.uint16)
@@ -270,7 +288,7 @@ def persistence_layers(layer: int, m: int):
 
 
 def compress(qwin_bits, k_bits, v_bits, budget, params: Params | None = None,
-             threads: int | None = None, units=None, keep_scores=False):
+             threads: int | None = None, units=None, keep_scores=False, adaptive_alpha=None):
     """The whole compression step on the host.
 
     qwin_bits [R, Ly, Hq, W, d], k_bits / v_bits [R, Ly, Hkv, N, d] are bf16
@@ -279,7 +297,9 @@ def compress(qwin_bits, k_bits, v_bits, budget, params: Params | None = None,
     the persistence term needs are then computed as well.
 
     ``budget`` is one budget for every layer or a sequence of per-layer
-    budgets (window included).
+    budgets (window included).  With ``adaptive_alpha`` the kept sets of a
+    (request, layer) are chosen jointly over its heads (select_adaptive);
+    ``units`` must then list whole layers (every head).
 
     Returns a dict keyed by (r, l, h) with 'idx', 'gap', 'lambda', 'Kc', 'Vc'
     and, when keep_scores, the score arrays of ``score_unit``.
@@ -317,7 +337,7 @@ def compress(qwin_bits, k_bits, v_bits, budget, params: Params | None = None,
             entry = {"idx": idx, "gap": gap, "lambda": sc["lambda"],
                      "Kc": gather(k_bits[r, l, h], idx),
                      "Vc": gather(v_bits[r, l, h], idx)}
-            if keep_scores:
+            if keep_scores or adaptive_alpha is not None:
                 entry.update(sc)
             res[(r, l, h)] = entry
         return res
@@ -327,4 +347,14 @@ def compress(qwin_bits, k_bits, v_bits, budget, params: Params | None = None,
     with ThreadPoolExecutor(max_workers=threads) as ex:
         for part in ex.map(run_chain, list(chains)):
             out.update(part)
+    if adaptive_alpha is not None:
+        layers_seen = sorted({(r, l) for (r, l, h) in out})
+        for (r, l) in layers_seen:
+            S = np.stack([out[(r, l, h)]["S"] for h in range(Hkv)])
+            kept = select_adaptive(S, W, layer_budget(l), adaptive_alpha, params)
+            for h in range(Hkv):
+                e = out[(r, l, h)]
+                e["idx"] = kept[h]
+                e["Kc"] = gather(k_bits[r, l, h], kept[h])
+                e["Vc"] = gather(v_bits[r, l, h], kept[h])
     return out

@@ -333,3 +333,46 @@ void bo_pyramid_budgets(int layers, int window, int budget, int beta, int* out)
         out[l] = K_min + (int)rise + window;
     }
 }
+
+/* (score desc, head asc, position asc) over the flattened (head, position)
+ * pairs; the flattened index h * n + i carries both tie-breaks. */
+int bo_select_adaptive(const double* S, int H, int N, int W, int budget, double alpha,
+                       const bo_params* p, int32_t* idx, int32_t* counts)
+{
+    if (H < 1 || N < 1 || W < 1 || W > N || budget < 0 || alpha < 0.0 || alpha > 1.0) return -1;
+    if (p->keep_window && budget < W) return -1;
+    int n_cand, keep;
+    bo_sizes(N, W, budget, p, &n_cand, &keep);
+    const int g = (int)floor(alpha * (double)keep);
+    char* taken = (char*)calloc((size_t)H * (size_t)(n_cand > 0 ? n_cand : 1), 1);
+    int32_t* order = (int32_t*)malloc(sizeof(int32_t) * (size_t)(n_cand > 0 ? n_cand : 1));
+    /* each head's guaranteed share */
+    for (int h = 0; h < H; ++h) {
+        bo_rank_topk(S + (size_t)h * N, n_cand, n_cand, order);
+        for (int j = 0; j < g && j < n_cand; ++j) taken[(size_t)h * n_cand + order[j]] = 1;
+    }
+    /* the rest, jointly over all heads */
+    const long total = (long)H * n_cand;
+    double* rest = (double*)malloc(sizeof(double) * (size_t)(total > 0 ? total : 1));
+    for (int h = 0; h < H; ++h)
+        for (int i = 0; i < n_cand; ++i)
+            rest[(size_t)h * n_cand + i] = taken[(size_t)h * n_cand + i] ? -INFINITY
+                                                                        : S[(size_t)h * N + i];
+    long R = (long)H * keep - (long)H * (g < n_cand ? g : n_cand);
+    int32_t* jorder = (int32_t*)malloc(sizeof(int32_t) * (size_t)(total > 0 ? total : 1));
+    bo_rank_topk(rest, (int)total, (int)total, jorder);
+    for (long j = 0; j < R && j < total; ++j) taken[jorder[j]] = 1;
+    for (int h = 0; h < H; ++h) {
+        int c = 0;
+        for (int i = 0; i < n_cand; ++i)
+            if (taken[(size_t)h * n_cand + i]) idx[(size_t)h * N + c++] = i;
+        if (p->keep_window)
+            for (int i = N - W; i < N; ++i) idx[(size_t)h * N + c++] = i;
+        counts[h] = c;
+    }
+    free(taken);
+    free(order);
+    free(rest);
+    free(jorder);
+    return 0;
+}

@@ -102,6 +102,18 @@ int bo_select(const double* S, int N, int W, int budget, const bo_params* p,
  * the layers together keep at most layers x K candidates. */
 void bo_pyramid_budgets(int layers, int window, int budget, int beta, int* out);
 
+/* AdaKV-style adaptive per-head budgets for one (request, layer), the base
+ * compressor of Sec. 5 / App. B that spreads a layer's budget over its heads.
+ * S [H][N] holds each head's final score (Eq. 16) over its candidates.  With
+ * K = budget - W per head on average, every head first keeps its own top
+ * g = floor(alpha K) candidates; the remaining H K - H g slots go to the best
+ * remaining candidates of all heads together (larger score first, ties to
+ * the lower head, then the lower position).  Head h's kept positions, in
+ * ascending order followed by the window, are written to idx + h * N;
+ * counts[h] receives their number.  Returns 0, or -1 on bad arguments. */
+int bo_select_adaptive(const double* S, int H, int N, int W, int budget, double alpha,
+                       const bo_params* p, int32_t* idx, int32_t* counts);
+
 /* Compacted cache: out[j] = x[idx[j]] row-wise, d values per row, bitwise. */
 void bo_gather(const uint16_t* x, int N, int d, const int32_t* idx,
                int count, uint16_t* out);

@@ -27,7 +27,8 @@ EXPORTS = ("bacon_default_params", "bacon_init", "bacon_destroy", "bacon_last_er
            "bacon_score_layer", "bacon_select", "bacon_compact",
            "bacon_compress_all_layers", "bacon_compress_host", "bacon_get_scores",
            "bacon_profile_enable", "bacon_profile_read", "bacon_window_scores_noalloc",
-           "bacon_compress_layer_budgets", "bacon_pyramid_budgets", "bacon_sync")
+           "bacon_compress_layer_budgets", "bacon_pyramid_budgets",
+           "bacon_compress_adaptive", "bacon_sync")
 PROFILE_STAGES = ("window_stats", "window_combine", "window_scores", "calibrate_select",
                   "gather")
 
@@ -87,13 +88,18 @@ def load() -> ctypes.CDLL:
                                                  ctypes.POINTER(_int), ctypes.POINTER(_vp),
                                                  ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp]
     lib.bacon_pyramid_budgets.argtypes = [_int, _int, _int, _int, ctypes.POINTER(_int)]
+    lib.bacon_compress_adaptive.argtypes = [_vp, _int, ctypes.POINTER(_vp), ctypes.POINTER(_vp),
+                                            ctypes.POINTER(_vp), _int, _int, ctypes.c_float,
+                                            ctypes.POINTER(_vp), ctypes.POINTER(_vp),
+                                            ctypes.POINTER(_vp), _vp, _vp]
     lib.bacon_pyramid_budgets.restype = None
     lib.bacon_window_scores_noalloc.argtypes = [_int, _int, _int, _int, _vp, _vp, _int, _vp,
                                                 _vp, _vp, _vp]
     lib.bacon_profile_enable.argtypes = [_vp, _int]
     lib.bacon_profile_read.argtypes = [_vp, ctypes.POINTER(ctypes.c_double),
                                        ctypes.POINTER(_int), _int]
-    for name in ("bacon_compress_layer_budgets", "bacon_window_scores_noalloc",
+    for name in ("bacon_compress_adaptive", "bacon_compress_layer_budgets",
+                 "bacon_window_scores_noalloc",
                  "bacon_profile_enable", "bacon_profile_read",
                  "bacon_init", "bacon_state_create", "bacon_state_reset", "bacon_score_layer",
                  "bacon_select", "bacon_compact", "bacon_compress_all_layers",
@@ -223,6 +229,26 @@ class Context:
                                                    tix, _stream_ptr(stream)))
         self._last_units, self._last_N = R * Ly * self.kv_heads, N
         return ko, vo, ix
+
+    def compress_adaptive(self, qwin, k, v, budget, alpha=0.2, stream=None):
+        """AdaKV-style head budgets.  Returns (k_out, v_out, idx, counts):
+        k_out/v_out [R, layers, Hkv * kept, d] and idx [R, layers, Hkv * kept]
+        flat per layer (heads in order), counts [R, layers, Hkv]."""
+        R, Ly, Hq, W, d = qwin.shape
+        N = k.shape[3]
+        kept = min(budget, N)
+        ko = torch.empty((R, Ly, self.kv_heads * kept, d), dtype=k.dtype, device=k.device)
+        vo = torch.empty_like(ko)
+        ix = torch.empty((R, Ly, self.kv_heads * kept), dtype=torch.int32, device=k.device)
+        counts = torch.empty((R, Ly, self.kv_heads), dtype=torch.int32, device=k.device)
+        pairs = [(r, l) for r in range(R) for l in range(Ly)]
+        tq, tk, tv, tko, tvo, tix = (_ptr_array([t[r, l].data_ptr() for r, l in pairs])
+                                     for t in (qwin, k, v, ko, vo, ix))
+        _check(load().bacon_compress_adaptive(self.handle, R, tq, tk, tv, N, budget,
+                                              float(alpha), tko, tvo, tix, counts.data_ptr(),
+                                              _stream_ptr(stream)))
+        self._last_units, self._last_N = R * Ly * self.kv_heads, N
+        return ko, vo, ix, counts
 
     def compress_host(self, qwin, k, v, budget, k_out=None, v_out=None, idx_out=None,
                       stream=None):

@@ -2,6 +2,7 @@
 // and the launch sequence of the compression step.
 #include <cstdarg>
 #include <cstdio>
+#include <cmath>
 #include <cstring>
 #include <new>
 #include <string>
@@ -275,10 +276,15 @@ struct StageEvents {
 
 // The whole step.  layer_budget[l] is the budget of layer l (window
 // included); idx[pair] receives the pair's [Hkv][min(budget, N)] positions.
+// With adaptive = true (uniform budget), the heads of each layer share the
+// budget (AdaKV-style, g = guaranteed candidates per head first): idx[pair]
+// and the K/V outputs are flat per pair, heads in order, with per-head kept
+// counts in `counts`.
 bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const void* const* k,
                              const void* const* v, int N, const int* layer_budget,
                              void* const* ko, void* const* vo, int32_t* const* idx,
-                             cudaStream_t st)
+                             cudaStream_t st, bool adaptive = false, int guaranteed = 0,
+                             int32_t* counts = nullptr)
 {
     const int pairs = R * c->layers;
     const Shape s = shape_of(c, c->layers, R, N);
@@ -321,12 +327,28 @@ bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const vo
     a.Bp = c->p.keep_scores ? c->Bp : nullptr;
     a.lambda = c->lam;
     a.compute_scores = 1;
-    a.do_select = 1;
-    a.write_S = c->p.keep_scores;
+    a.do_select = adaptive ? 0 : 1;
+    a.write_S = (c->p.keep_scores || adaptive) ? 1 : 0;
     a.err = c->err;
     BACON_CUDA(launch_calibrate_select(s, calib_of(c), a, st), "calibrate_select launch");
+    if (adaptive) {
+        AdaptArgs ad;
+        ad.S = c->S;
+        ad.budget = layer_budget[0];
+        ad.guaranteed = guaranteed;
+        for (int i = 0; i < pairs; ++i) {
+            ad.idx[i] = idx[i];
+            gt.kept[i] = c->hkv * (layer_budget[0] < N ? layer_budget[0] : N);
+        }
+        ad.counts = counts;
+        ad.err = c->err;
+        BACON_CUDA(launch_adaptive_select(s, c->p.keep_window, ad, st), "adaptive select launch");
+    }
     prof.mark(4);
-    BACON_CUDA(launch_gather(gt, s, c->err, st), "gather launch");
+    if (adaptive)
+        BACON_CUDA(launch_gather_flat(gt, s, counts, c->err, st), "gather launch");
+    else
+        BACON_CUDA(launch_gather(gt, s, c->err, st), "gather launch");
     prof.mark(5);
     prof.commit();
     c->last_units = s.units;
@@ -439,7 +461,7 @@ bacon_status bacon_init(bacon_ctx** out, int layers, int kv_heads, int q_heads, 
     if (e == cudaSuccess) e = dalloc(&c->B, tok);
     if (e == cudaSuccess) e = dalloc(&c->Q, tok);
     if (e == cudaSuccess) e = dalloc(&c->E, tok);
-    if (e == cudaSuccess) e = dalloc(&c->S, prm.keep_scores ? tok : 0);
+    if (e == cudaSuccess) e = dalloc(&c->S, tok);
     if (e == cudaSuccess) e = dalloc(&c->V, prm.keep_scores ? tok : 0);
     if (e == cudaSuccess) e = dalloc(&c->Bp, prm.keep_scores ? tok : 0);
     if (e == cudaSuccess) e = dalloc(&c->lam, c->unit_cap);
@@ -682,6 +704,38 @@ bacon_status bacon_compress_layer_budgets(bacon_ctx* ctx, int requests, const vo
     DeviceGuard dg(ctx->device);
     return compress_device(ctx, requests, q_win, k, v, seq_len, layer_budgets, k_out, v_out,
                            idx_out, static_cast<cudaStream_t>(stream));
+}
+
+bacon_status bacon_compress_adaptive(bacon_ctx* ctx, int requests, const void* const* q_win,
+                                     const void* const* k, const void* const* v, int seq_len,
+                                     int budget, float alpha, void* const* k_out,
+                                     void* const* v_out, int32_t* const* idx_out,
+                                     int32_t* counts_out, bacon_stream stream)
+{
+    g_last_error.clear();
+    if (!ctx) return fail(BACON_EINVAL, "null context");
+    if (requests < 1 || requests > ctx->p.max_requests)
+        return fail(BACON_EINVAL, "requests %d outside [1, %d]", requests, ctx->p.max_requests);
+    if (!(alpha >= 0.f && alpha <= 1.f)) return fail(BACON_EINVAL, "alpha %g outside [0, 1]", (double)alpha);
+    bacon_status rc = check_seq(ctx, seq_len, budget);
+    if (rc != BACON_OK) return rc;
+    rc = check_pointer_arrays(ctx, requests * ctx->layers, q_win, k, v, k_out, v_out);
+    if (rc != BACON_OK) return rc;
+    if (!idx_out || !counts_out || !aligned16(counts_out)) return fail(BACON_EINVAL, "null index or count array");
+    for (int i = 0; i < requests * ctx->layers; ++i)
+        if (!idx_out[i] || !aligned16(idx_out[i]))
+            return fail(BACON_EINVAL, "index pointer of pair %d must be a 16-byte aligned device pointer", i);
+    const int win = ctx->p.keep_window ? ctx->W : 0;
+    if (adaptive_smem(ctx->hkv, seq_len - win) > 200 * 1024)
+        return fail(BACON_EUNSUPPORTED, "kv_heads x candidates = %d exceeds the adaptive selection's %d",
+                    ctx->hkv * (seq_len - win), 200 * 1024);
+    const int kept = budget < seq_len ? budget : seq_len;
+    const int guaranteed = (int)floor((double)alpha * (double)(kept - win));
+    DeviceGuard dg(ctx->device);
+    std::vector<int> budgets(ctx->layers, budget);
+    return compress_device(ctx, requests, q_win, k, v, seq_len, budgets.data(), k_out, v_out,
+                           idx_out, static_cast<cudaStream_t>(stream), true, guaranteed,
+                           counts_out);
 }
 
 void bacon_pyramid_budgets(int layers, int window, int budget, int beta, int* out)

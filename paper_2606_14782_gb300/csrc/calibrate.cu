@@ -6,79 +6,17 @@
 //   S = B~ + lambda V                                 (Eq. 16)
 //   the K best candidates by S, ascending, then the window (Eq. 17)
 // Both "best k" sets use one order: larger value first, equal values ->
-// lower position first.  They are found by a 4 x 8-bit radix select on the
-// order-preserving float keys, then an index-ordered block scan resolves the
-// ties at the threshold and emits the kept positions in ascending order.
+// lower position first (select.cuh: radix select, then index-ordered
+// warp-segmented sweeps that resolve ties and emit ascending positions).
 #include "common.cuh"
+#include "select.cuh"
 
 namespace bacon {
 namespace {
 
+using namespace sel;
+
 constexpr int kThreads = 1024;
-
-struct SelectResult {
-    uint32_t tau;   // key of the k-th best element
-    int need;       // how many elements with key == tau are taken
-};
-
-// Block-wide: k-th largest key over vals[0, n) (1 <= k <= n).  Every thread
-// returns the same result.
-__device__ SelectResult radix_select(const float* vals, int n, int k, int* hist, int* bcast)
-{
-    uint32_t prefix = 0, mask = 0;
-    int remaining = k;
-    for (int shift = 24; shift >= 0; shift -= 8) {
-        for (int b = threadIdx.x; b < 256; b += blockDim.x) hist[b] = 0;
-        __syncthreads();
-        // warp-aggregated: lanes that fall into the same bin add once together
-        const int n_round = (n + 31) & ~31;
-        for (int i = threadIdx.x; i < n_round; i += blockDim.x) {
-            const bool in = i < n;
-            const uint32_t key = in ? float_key(vals[i]) : 0u;
-            const bool hit = in && (key & mask) == prefix;
-            const int bin = hit ? (int)((key >> shift) & 255u) : -1;
-            const uint32_t peers = __match_any_sync(0xffffffffu, bin);
-            if (hit && (threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
-        }
-        __syncthreads();
-        if (threadIdx.x < 32) {
-            // warp 0: bins high to low; find the bin where the running count
-            // from the top reaches `remaining`
-            const int lane = threadIdx.x;
-            int cum = 0, found_bin = -1, found_rem = 0;
-            for (int base = 255; base >= 0 && found_bin < 0; base -= 32) {
-                const int b = base - lane;
-                const int c = hist[b];
-                // inclusive scan from the top (lane 0 = highest bin)
-                int incl = c;
-#pragma unroll
-                for (int o = 1; o < 32; o <<= 1) {
-                    const int y = __shfl_up_sync(0xffffffffu, incl, o);
-                    if (lane >= o) incl += y;
-                }
-                const bool hit = cum + incl >= remaining;
-                const uint32_t ballot = __ballot_sync(0xffffffffu, hit);
-                if (ballot) {
-                    const int first = __ffs(ballot) - 1;
-                    const int excl = __shfl_sync(0xffffffffu, incl - c, first);
-                    found_bin = base - first;
-                    found_rem = remaining - (cum + excl);
-                }
-                cum += __shfl_sync(0xffffffffu, incl, 31);
-            }
-            if (lane == 0) {
-                bcast[0] = found_bin;
-                bcast[1] = found_rem;
-            }
-        }
-        __syncthreads();
-        prefix |= (uint32_t)bcast[0] << shift;
-        mask |= 255u << shift;
-        remaining = bcast[1];
-        __syncthreads();
-    }
-    return {prefix, remaining};
-}
 
 // Block-wide fp32 sum by a shuffle tree (pairwise, so the rounding error
 // grows with log2 of the count).  FP64 is avoided: its rate on this part is
@@ -119,84 +57,6 @@ __device__ __forceinline__ void stage(float* dst, const float* src, int n)
         for (int k = 0; k < 4; ++k)
             if (i + k * (int)blockDim.x < n4) d4[i + k * blockDim.x] = v[k];
     }
-}
-
-// Index-ordered sweeps over vals[0, n): warp w owns the contiguous segment
-// [lo, hi) and its lanes take consecutive elements, so shared-memory reads
-// are conflict-free while ballots keep the index order inside a warp.
-struct Segment {
-    int lo, hi;
-};
-
-__device__ __forceinline__ Segment warp_segment(int n)
-{
-    const int nw = blockDim.x >> 5;
-    const int per = ((n + nw - 1) / nw + 31) & ~31;
-    const int lo = min(n, (int)(threadIdx.x >> 5) * per);
-    return {lo, min(n, lo + per)};
-}
-
-__device__ __forceinline__ int warp_sum(int v)
-{
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    return v;
-}
-
-// Exclusive scan of one value per warp (lane 0's `v`), returned to every lane.
-__device__ int warp_exclusive_scan(int v, int* warp_sums, int* total)
-{
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    if (lane == 0) warp_sums[warp] = v;
-    __syncthreads();
-    if (warp == 0) {
-        const int nw = blockDim.x >> 5;
-        const int w = lane < nw ? warp_sums[lane] : 0;
-        int incl = w;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, incl, o);
-            if (lane >= o) incl += y;
-        }
-        if (lane < nw) warp_sums[lane] = incl - w;
-        if (lane == 31) *total = incl;
-    }
-    __syncthreads();
-    const int r = warp_sums[warp];
-    __syncthreads();
-    return r;
-}
-
-// Walks this warp's segment in index order; calls f(i, in) for every index
-// with in = membership in the k best (key > tau, or key == tau among the
-// first `need` equal keys).  eq_before = equal keys before the segment.
-template <typename F>
-__device__ __forceinline__ void walk_topk(const float* vals, Segment sg, SelectResult sel,
-                                          int eq_before, F f)
-{
-    const int lane = threadIdx.x & 31;
-    const uint32_t lt = (1u << lane) - 1u;
-    int running = eq_before;
-    for (int base = sg.lo; base < sg.hi; base += 32) {
-        const int i = base + lane;
-        const bool valid = i < sg.hi;
-        const uint32_t key = valid ? float_key(vals[i]) : 0u;
-        const bool eq = valid && key == sel.tau;
-        const uint32_t ball = __ballot_sync(0xffffffffu, eq);
-        const int rank = running + __popc(ball & lt);
-        const bool in = valid && (key > sel.tau || (eq && rank < sel.need));
-        f(i, valid, in);
-        running += __popc(ball);
-    }
-}
-
-// Equal-to-threshold keys before this warp's segment.
-__device__ int eq_before_segment(const float* vals, Segment sg, uint32_t tau, int* warp_sums,
-                                 int* total)
-{
-    int eq = 0;
-    for (int i = sg.lo + (threadIdx.x & 31); i < sg.hi; i += 32) eq += float_key(vals[i]) == tau;
-    return warp_exclusive_scan(warp_sum(eq), warp_sums, total);
 }
 
 __global__ void __launch_bounds__(kThreads)

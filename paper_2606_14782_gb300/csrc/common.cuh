@@ -92,6 +92,23 @@ cudaError_t launch_calibrate_select(const Shape& s, const Calib& c, const CalibA
 // Dynamic shared memory of the calibration kernel for N tokens.
 size_t calibrate_smem(int N);
 
+// AdaKV-style selection over the heads of each (request, layer).
+struct AdaptArgs {
+    const float* S;              // [units][N] final scores (0 off-candidates)
+    int budget;                  // average per-head budget (window included)
+    int guaranteed;              // g = floor(alpha K) candidates per head first
+    int32_t* idx[kMaxPairs];     // per pair: flat [Hkv * kept] positions, heads in order
+    int32_t* counts;             // [pairs][Hkv] kept per head (window included)
+    int* err;
+};
+cudaError_t launch_adaptive_select(const Shape& s, int keep_window, const AdaptArgs& a,
+                                   cudaStream_t st);
+// Dynamic shared memory of the adaptive selection (one byte per candidate).
+size_t adaptive_smem(int kv_heads, int n_cand);
+// Gather into the flat per-layer layout of the adaptive selection.
+cudaError_t launch_gather_flat(const GatherTable& tab, const Shape& s, const int32_t* counts,
+                               int* err, cudaStream_t st);
+
 // Gather of the kept K/V rows (kept counts may differ between pairs).
 cudaError_t launch_gather(const GatherTable& tab, const Shape& s, int* err, cudaStream_t st);
 

@@ -76,12 +76,13 @@ def compare(wl, x, budget, gpu, orc, report=None):
     return swaps
 
 
-def oracle_run(wl, x, budget, units=None, **kw):
+def oracle_run(wl, x, budget, units=None, adaptive_alpha=None, **kw):
     qb = workloads.bf16_bits(x.qwin)
     kb = workloads.bf16_bits(x.k)
     vb = workloads.bf16_bits(x.v)
     p = oracle_params(pool_kernel=wl.pool, **kw)
-    res = oracle.compress(qb, kb, vb, budget, p, threads=THREADS, units=units, keep_scores=True)
+    res = oracle.compress(qb, kb, vb, budget, p, threads=THREADS, units=units, keep_scores=True,
+                          adaptive_alpha=adaptive_alpha)
     res["_keep_window"] = p.keep_window
     return res
 
@@ -357,3 +358,74 @@ def test_uniform_layer_budgets_match_whole_step():
             assert np.array_equal(ix[r][l].cpu().numpy(), whole["idx"][r, l])
             assert torch.equal(ko[r][l].cpu(), whole["Kc"][r, l])
     ctx.close()
+
+
+# ------------------------------------------------ adaptive head budgets (AdaKV)
+
+def _head_threshold(S_cand, k):
+    order = np.lexsort((np.arange(S_cand.size), -S_cand))
+    return S_cand[order[k - 1]] if k > 0 else np.inf
+
+
+@pytest.mark.parametrize("name,budget,alpha", [("tiny", 64, 0.2), ("tiny", 64, 1.0),
+                                               ("llava", 128, 0.2), ("qwen-img", 256, 0.0)])
+def test_adaptive_head_budgets_parity(name, budget, alpha):
+    base = workloads.CONFIGS[name]
+    wl = base.with_(layers=min(3, base.layers))
+    x = workloads.generate(wl, seed=8, device="cuda")
+    N, W, H = wl.seq_len, wl.window, wl.kv_heads
+    p = bacon.default_params(keep_scores=1, max_seq_len=N, max_requests=wl.requests)
+    ctx = bacon.Context(wl.layers, H, wl.q_heads, wl.head_dim, wl.window, wl.pool, budget,
+                        params=p)
+    ko, vo, ix, counts = ctx.compress_adaptive(x.qwin, x.k, x.v, budget, alpha)
+    ctx.sync()
+    S = ctx.scores("S").cpu().numpy().reshape(wl.requests, wl.layers, H, N)
+    ctx.close()
+    ko, vo, ix, counts = ko.cpu(), vo.cpu(), ix.cpu().numpy(), counts.cpu().numpy()
+    orc = oracle_run(wl, x, budget, adaptive_alpha=alpha)
+    kb = workloads.bf16_bits(x.k)
+    vb = workloads.bf16_bits(x.v)
+    K = min(budget, N) - W
+    g = int(np.floor(alpha * K))
+    swaps = 0
+    for r in range(wl.requests):
+        for l in range(wl.layers):
+            cnt = counts[r, l]
+            assert cnt.sum() == H * min(budget, N) and (cnt >= g + W).all()
+            off = np.concatenate([[0], np.cumsum(cnt)])
+            gpu_sets, orc_sets, S_orc = set(), set(), {}
+            thresholds = []
+            for h in range(H):
+                o = orc[(r, l, h)]
+                check_scores(f"S {(r, l, h)}", S[r, l, h], o["S"])
+                seg = ix[r, l, off[h]:off[h + 1]]
+                assert np.all(np.diff(seg) > 0)
+                assert np.array_equal(seg[-W:], np.arange(N - W, N))
+                Kc = ko[r, l, off[h]:off[h + 1]].view(torch.int16).numpy().view(np.uint16)
+                Vc = vo[r, l, off[h]:off[h + 1]].view(torch.int16).numpy().view(np.uint16)
+                assert np.array_equal(Kc, kb[r, l, h][seg]) and np.array_equal(Vc, vb[r, l, h][seg])
+                gpu_sets |= {(h, int(i)) for i in seg[:-W]}
+                orc_sets |= {(h, int(i)) for i in o["idx"][:-W]}
+                S_orc.update({(h, i): o["S"][i] for i in range(N - W)})
+                thresholds.append(_head_threshold(o["S"][:N - W], g))
+            # joint threshold: the lowest oracle score among the oracle's picks
+            thresholds.append(min(S_orc[t] for t in orc_sets))
+            for t in gpu_sets ^ orc_sets:
+                sv = S_orc[t]
+                assert min(abs(sv - th) for th in thresholds) <= 1e-5 + 2e-3 * abs(sv), (r, l, t, sv)
+            swaps += len(gpu_sets - orc_sets)
+    assert swaps <= max(2, wl.requests * wl.layers * H * K // 500)
+
+
+def test_adaptive_alpha_one_equals_uniform():
+    wl = workloads.CONFIGS["tiny"].with_(layers=3)
+    x = workloads.generate(wl, seed=9, device="cuda")
+    whole = run_gpu(wl, x, 64)
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool, 64,
+                        max_seq_len=wl.seq_len, max_requests=1)
+    ko, vo, ix, counts = ctx.compress_adaptive(x.qwin, x.k, x.v, 64, 1.0)
+    ctx.sync()
+    ctx.close()
+    assert (counts.cpu().numpy() == 64).all()
+    assert np.array_equal(ix.cpu().numpy().reshape(whole["idx"].shape), whole["idx"])
+    assert torch.equal(ko.cpu().reshape(whole["Kc"].shape), whole["Kc"])

@@ -510,3 +510,61 @@ def test_compress_accepts_layer_budgets():
     one = oracle.compress(qb, kb, vb, int(budgets[1]), oracle.Params(), threads=2,
                           units=[(0, 1, 2)])
     assert np.array_equal(one[(0, 1, 2)]["idx"], res[(0, 1, 2)]["idx"])
+
+
+# ---------------------------------------------- AdaKV adaptive head budgets
+
+def test_adaptive_alpha_one_is_per_head_topk():
+    rng = np.random.default_rng(21)
+    H, N, W, budget = 3, 60, 6, 20
+    S = rng.random((H, N))
+    S[:, N - W:] = 0.0
+    kept = oracle.select_adaptive(S, W, budget, 1.0, Params())
+    for h in range(H):
+        want, _ = oracle.select(S[h], N, W, budget, Params())
+        assert np.array_equal(kept[h], want)
+
+
+def test_adaptive_single_head_is_topk():
+    rng = np.random.default_rng(22)
+    S = rng.random((1, 50))
+    for alpha in (0.0, 0.2, 0.5):
+        kept = oracle.select_adaptive(S, 5, 17, alpha, Params())
+        want, _ = oracle.select(S[0], 50, 5, 17, Params())
+        assert np.array_equal(kept[0], want)
+
+
+def test_adaptive_hand_worked():
+    # two heads, 6 candidates each + window 2, budget 5 -> K = 3, H K = 6;
+    # alpha 1/3 -> g = 1 guaranteed per head, 4 slots jointly.
+    S = np.array([[9, 8, 7, 6, 0.5, 0.4, 0, 0],
+                  [5, 1, 1, 1, 1, 1, 0, 0]], dtype=float)
+    kept = oracle.select_adaptive(S, 2, 5, 1 / 3, Params())
+    # guaranteed: head 0 -> 0 (9), head 1 -> 0 (5); jointly the best of the
+    # rest: 8, 7, 6 (head 0) then the first 1 of head 1 (ties: lower position)
+    assert kept[0].tolist() == [0, 1, 2, 3, 6, 7]
+    assert kept[1].tolist() == [0, 1, 6, 7]
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_adaptive_invariants(seed):
+    rng = np.random.default_rng(30 + seed)
+    H, N, W, budget, alpha = 4, 80, 8, 24, 0.25
+    S = rng.integers(0, 6, (H, N)).astype(float)  # ties everywhere
+    kept = oracle.select_adaptive(S, W, budget, alpha, Params())
+    K, g = budget - W, int(alpha * (budget - W))
+    cand = [k[:-W] for k in kept]
+    assert sum(len(c) for c in cand) == H * K
+    assert all(len(c) >= g for c in cand)
+    for k in kept:
+        assert np.all(np.diff(k) > 0) and np.array_equal(k[-W:], np.arange(N - W, N))
+    # every jointly chosen candidate dominates every candidate left out
+    # (score desc, head asc, position asc), guaranteed ones aside
+    guaranteed = set()
+    for h in range(H):
+        for i in oracle.rank_topk(S[h, :N - W], g):
+            guaranteed.add((h, int(i)))
+    chosen = {(h, int(i)) for h in range(H) for i in cand[h]} - guaranteed
+    left = {(h, i) for h in range(H) for i in range(N - W)} - {(h, int(i)) for h in range(H) for i in cand[h]}
+    key = lambda t: (-S[t[0], t[1]], t[0], t[1])
+    assert max(key(t) for t in chosen) < min(key(t) for t in left)
