@@ -104,6 +104,9 @@ struct bacon_ctx {
     cudaEvent_t maps_ev = nullptr;
     std::vector<const void*> map_key;
     int map_key_N = -1;
+    // host-buffer path: copy streams and per-request events
+    cudaStream_t h2d = nullptr, d2h = nullptr;
+    std::vector<cudaEvent_t> ev_in, ev_done;
     // per-kernel timing (bacon_profile_enable)
     int prof_on = 0;
     std::vector<cudaEvent_t> ev_free;
@@ -225,6 +228,13 @@ TcArgs tc_args(const Shape& s, const CUtensorMap* kmaps, const CUtensorMap* qmap
 
 void free_ctx_buffers(bacon_ctx* c)
 {
+    for (cudaEvent_t e : c->ev_in) cudaEventDestroy(e);
+    for (cudaEvent_t e : c->ev_done) cudaEventDestroy(e);
+    c->ev_in.clear();
+    c->ev_done.clear();
+    if (c->h2d) cudaStreamDestroy(c->h2d);
+    if (c->d2h) cudaStreamDestroy(c->d2h);
+    c->h2d = c->d2h = nullptr;
     if (c->maps_ev) cudaEventDestroy(c->maps_ev);
     if (c->h_maps) cudaFreeHost(c->h_maps);
     if (c->d_maps) cudaFree(c->d_maps);
@@ -284,10 +294,19 @@ bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const vo
                              const void* const* v, int N, const int* layer_budget,
                              void* const* ko, void* const* vo, int32_t* const* idx,
                              cudaStream_t st, bool adaptive = false, int guaranteed = 0,
-                             int32_t* counts = nullptr)
+                             int32_t* counts = nullptr, size_t unit0 = 0)
 {
     const int pairs = R * c->layers;
     const Shape s = shape_of(c, c->layers, R, N);
+    // this call's slice of the scratch starts at unit `unit0`
+    const int chunks = (N + kTcChunkTokens - 1) / kTcChunkTokens;
+    float* B = c->B + unit0 * N;
+    float* Q = c->Q + unit0 * N;
+    float* E = c->E + unit0 * N;
+    float* S = c->S + unit0 * N;
+    float* lam = c->lam + unit0;
+    float* lse2 = c->lse2 + unit0 * c->rows;
+    float2* partial = c->partial + unit0 * chunks * c->rows;
 
     GatherTable gt;
     CalibArgs a;
@@ -306,26 +325,25 @@ bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const vo
     bacon_status rc = upload_maps(c, c->d_maps, c->h_maps, c->maps_ev, c->map_key, c->map_key_N,
                                   kMaxPairs, pairs, q, k, N, st);
     if (rc != BACON_OK) return rc;
-    const TcArgs ta = tc_args(s, c->d_maps, c->d_maps + kMaxPairs, c->partial, c->lse2, c->B,
-                              c->Q, c->E, c->err);
+    const TcArgs ta = tc_args(s, c->d_maps, c->d_maps + kMaxPairs, partial, lse2, B, Q, E, c->err);
     StageEvents prof(c, st);
     prof.mark(0);
     BACON_CUDA(launch_window_stats_tc(ta, st), "window_stats launch");
     prof.mark(1);
-    BACON_CUDA(launch_window_combine(s, ta.chunks, c->partial, c->lse2, st), "window_combine launch");
+    BACON_CUDA(launch_window_combine(s, ta.chunks, partial, lse2, st), "window_combine launch");
     prof.mark(2);
     BACON_CUDA(launch_window_scores_tc(ta, st), "window_scores launch");
     prof.mark(3);
 
-    a.B = c->B;
-    a.Ering = c->E;
+    a.B = B;
+    a.Ering = E;
     a.ring = c->layers;
     a.ring_req_stride = (long long)c->layers * c->hkv * N;
     a.layer0 = 0;
-    a.S = c->S;
-    a.V = c->p.keep_scores ? c->V : nullptr;
-    a.Bp = c->p.keep_scores ? c->Bp : nullptr;
-    a.lambda = c->lam;
+    a.S = S;
+    a.V = c->p.keep_scores ? c->V + unit0 * N : nullptr;
+    a.Bp = c->p.keep_scores ? c->Bp + unit0 * N : nullptr;
+    a.lambda = lam;
     a.compute_scores = 1;
     a.do_select = adaptive ? 0 : 1;
     a.write_S = (c->p.keep_scores || adaptive) ? 1 : 0;
@@ -333,7 +351,7 @@ bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const vo
     BACON_CUDA(launch_calibrate_select(s, calib_of(c), a, st), "calibrate_select launch");
     if (adaptive) {
         AdaptArgs ad;
-        ad.S = c->S;
+        ad.S = S;
         ad.budget = layer_budget[0];
         ad.guaranteed = guaranteed;
         for (int i = 0; i < pairs; ++i) {
@@ -351,7 +369,7 @@ bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const vo
         BACON_CUDA(launch_gather(gt, s, c->err, st), "gather launch");
     prof.mark(5);
     prof.commit();
-    c->last_units = s.units;
+    c->last_units = (int)unit0 + s.units;
     c->last_N = N;
     return BACON_OK;
 }
@@ -783,9 +801,37 @@ bacon_status bacon_compress_host(bacon_ctx* ctx, int requests, const void* q_win
     ctx->hout_cap = o_cap;
     if ((rc = grow(&ctx->hidx_buf, &ctx->hidx_cap, idx_count * 4, "indices")) != BACON_OK) return rc;
 
-    BACON_CUDA(cudaMemcpyAsync(ctx->hq_buf, q_win, q_pair * pairs * 2, cudaMemcpyHostToDevice, cs), "query upload");
-    BACON_CUDA(cudaMemcpyAsync(ctx->hk_buf, k, kv_pair * pairs * 2, cudaMemcpyHostToDevice, cs), "key upload");
-    BACON_CUDA(cudaMemcpyAsync(ctx->hv_buf, v, kv_pair * pairs * 2, cudaMemcpyHostToDevice, cs), "value upload");
+    if (!ctx->h2d) {
+        BACON_CUDA(cudaStreamCreateWithFlags(&ctx->h2d, cudaStreamNonBlocking), "copy stream");
+        BACON_CUDA(cudaStreamCreateWithFlags(&ctx->d2h, cudaStreamNonBlocking), "copy stream");
+    }
+    while ((int)ctx->ev_in.size() < requests) {
+        cudaEvent_t a = nullptr, b = nullptr;
+        BACON_CUDA(cudaEventCreateWithFlags(&a, cudaEventDisableTiming), "event");
+        BACON_CUDA(cudaEventCreateWithFlags(&b, cudaEventDisableTiming), "event");
+        ctx->ev_in.push_back(a);
+        ctx->ev_done.push_back(b);
+    }
+    // Requests are pipelined: every upload is queued on one copy stream, a
+    // request is compressed on the caller's stream as soon as its inputs have
+    // landed, and its outputs go back on a second copy stream while the next
+    // request computes.
+    const int L = ctx->layers;
+    const char* qh = static_cast<const char*>(q_win);
+    const char* kh = static_cast<const char*>(k);
+    const char* vh = static_cast<const char*>(v);
+    BACON_CUDA(cudaEventRecord(ctx->ev_done[0], cs), "event");  // uploads start after earlier work
+    BACON_CUDA(cudaStreamWaitEvent(ctx->h2d, ctx->ev_done[0], 0), "event wait");
+    for (int r = 0; r < requests; ++r) {
+        const size_t qb = q_pair * L * 2, kb = kv_pair * L * 2;
+        BACON_CUDA(cudaMemcpyAsync(static_cast<char*>(ctx->hq_buf) + r * qb, qh + r * qb, qb,
+                                   cudaMemcpyHostToDevice, ctx->h2d), "query upload");
+        BACON_CUDA(cudaMemcpyAsync(static_cast<char*>(ctx->hk_buf) + r * kb, kh + r * kb, kb,
+                                   cudaMemcpyHostToDevice, ctx->h2d), "key upload");
+        BACON_CUDA(cudaMemcpyAsync(static_cast<char*>(ctx->hv_buf) + r * kb, vh + r * kb, kb,
+                                   cudaMemcpyHostToDevice, ctx->h2d), "value upload");
+        BACON_CUDA(cudaEventRecord(ctx->ev_in[r], ctx->h2d), "event");
+    }
 
     const void* qs[kMaxPairs];
     const void* ks[kMaxPairs];
@@ -799,14 +845,30 @@ bacon_status bacon_compress_host(bacon_ctx* ctx, int requests, const void* q_win
         kos[i] = static_cast<uint16_t*>(ctx->hko_buf) + o_pair * i;
         vos[i] = static_cast<uint16_t*>(ctx->hvo_buf) + o_pair * i;
     }
-    std::vector<int> budgets(ctx->layers, budget);
+    std::vector<int> budgets(L, budget);
     int32_t* idx_pairs[kMaxPairs];
     for (int i = 0; i < pairs; ++i) idx_pairs[i] = ctx->hidx_buf + (size_t)i * ctx->hkv * kept;
-    rc = compress_device(ctx, requests, qs, ks, vs, seq_len, budgets.data(), kos, vos, idx_pairs, cs);
-    if (rc != BACON_OK) return rc;
-    BACON_CUDA(cudaMemcpyAsync(k_out, ctx->hko_buf, o_pair * pairs * 2, cudaMemcpyDeviceToHost, cs), "key download");
-    BACON_CUDA(cudaMemcpyAsync(v_out, ctx->hvo_buf, o_pair * pairs * 2, cudaMemcpyDeviceToHost, cs), "value download");
-    BACON_CUDA(cudaMemcpyAsync(idx_out, ctx->hidx_buf, idx_count * 4, cudaMemcpyDeviceToHost, cs), "index download");
+    for (int r = 0; r < requests; ++r) {
+        BACON_CUDA(cudaStreamWaitEvent(cs, ctx->ev_in[r], 0), "event wait");
+        rc = compress_device(ctx, 1, qs + r * L, ks + r * L, vs + r * L, seq_len, budgets.data(),
+                             kos + r * L, vos + r * L, idx_pairs + r * L, cs, false, 0, nullptr,
+                             (size_t)r * L * ctx->hkv);
+        if (rc != BACON_OK) return rc;
+        BACON_CUDA(cudaEventRecord(ctx->ev_done[r], cs), "event");
+        BACON_CUDA(cudaStreamWaitEvent(ctx->d2h, ctx->ev_done[r], 0), "event wait");
+        const size_t ob = o_pair * L * 2, ib = (size_t)L * ctx->hkv * kept * 4;
+        BACON_CUDA(cudaMemcpyAsync(static_cast<char*>(k_out) + r * ob,
+                                   static_cast<char*>(ctx->hko_buf) + r * ob, ob,
+                                   cudaMemcpyDeviceToHost, ctx->d2h), "key download");
+        BACON_CUDA(cudaMemcpyAsync(static_cast<char*>(v_out) + r * ob,
+                                   static_cast<char*>(ctx->hvo_buf) + r * ob, ob,
+                                   cudaMemcpyDeviceToHost, ctx->d2h), "value download");
+        BACON_CUDA(cudaMemcpyAsync(reinterpret_cast<char*>(idx_out) + r * ib,
+                                   reinterpret_cast<char*>(ctx->hidx_buf) + r * ib, ib,
+                                   cudaMemcpyDeviceToHost, ctx->d2h), "index download");
+    }
+    (void)idx_count;
+    BACON_CUDA(cudaStreamSynchronize(ctx->d2h), "host-path synchronisation");
     BACON_CUDA(cudaStreamSynchronize(cs), "host-path synchronisation");
     return bacon_sync(ctx, stream);
 }
