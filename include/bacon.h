@@ -166,6 +166,20 @@ bacon_status bacon_compress_layer_budgets(bacon_ctx* ctx, int requests,
                                           void* const* v_out, int32_t* const* idx_out,
                                           bacon_stream stream);
 
+/* The whole step when the caller's prefill attention already produced the
+ * softmax normalisers of the window rows (a fused attention kernel keeps
+ * the log-sum-exp of every query row; Eq. 1's rows need nothing else to be
+ * normalised), so the first pass over K is skipped.  lse is a HOST array of
+ * DEVICE pointers [request * layers + layer], each fp32 [Hq][W]: for window
+ * query w of query head g, ln sum_{i <= N-W+w} exp(q . k_i / sqrt(d)).
+ * Everything else, including outputs and errors, as bacon_compress_all_layers.
+ * Results equal that call's up to the rounding of the supplied values. */
+bacon_status bacon_compress_with_lse(bacon_ctx* ctx, int requests, const void* const* q_win,
+                                     const void* const* k, const void* const* v,
+                                     const float* const* lse, int seq_len, int budget,
+                                     void* const* k_out, void* const* v_out, int32_t* idx_out,
+                                     bacon_stream stream);
+
 /* The whole step with AdaKV-style adaptive head budgets (Sec. 5 / App. B:
  * the base compressor spreads a layer's budget over its kv-heads; BACON
  * supplies the score, Eq. 16, with K of Eq. 12 the average per-head budget).

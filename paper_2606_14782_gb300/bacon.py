@@ -28,7 +28,7 @@ EXPORTS = ("bacon_default_params", "bacon_init", "bacon_destroy", "bacon_last_er
            "bacon_compress_all_layers", "bacon_compress_host", "bacon_get_scores",
            "bacon_profile_enable", "bacon_profile_read", "bacon_window_scores_noalloc",
            "bacon_compress_layer_budgets", "bacon_pyramid_budgets",
-           "bacon_compress_adaptive", "bacon_sync")
+           "bacon_compress_adaptive", "bacon_compress_with_lse", "bacon_sync")
 PROFILE_STAGES = ("window_stats", "window_combine", "window_scores", "calibrate_select",
                   "gather")
 
@@ -88,6 +88,9 @@ def load() -> ctypes.CDLL:
                                                  ctypes.POINTER(_int), ctypes.POINTER(_vp),
                                                  ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp]
     lib.bacon_pyramid_budgets.argtypes = [_int, _int, _int, _int, ctypes.POINTER(_int)]
+    lib.bacon_compress_with_lse.argtypes = [_vp, _int, ctypes.POINTER(_vp), ctypes.POINTER(_vp),
+                                            ctypes.POINTER(_vp), ctypes.POINTER(_vp), _int, _int,
+                                            ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp, _vp]
     lib.bacon_compress_adaptive.argtypes = [_vp, _int, ctypes.POINTER(_vp), ctypes.POINTER(_vp),
                                             ctypes.POINTER(_vp), _int, _int, ctypes.c_float,
                                             ctypes.POINTER(_vp), ctypes.POINTER(_vp),
@@ -98,7 +101,8 @@ def load() -> ctypes.CDLL:
     lib.bacon_profile_enable.argtypes = [_vp, _int]
     lib.bacon_profile_read.argtypes = [_vp, ctypes.POINTER(ctypes.c_double),
                                        ctypes.POINTER(_int), _int]
-    for name in ("bacon_compress_adaptive", "bacon_compress_layer_budgets",
+    for name in ("bacon_compress_with_lse", "bacon_compress_adaptive",
+                 "bacon_compress_layer_budgets",
                  "bacon_window_scores_noalloc",
                  "bacon_profile_enable", "bacon_profile_read",
                  "bacon_init", "bacon_state_create", "bacon_state_reset", "bacon_score_layer",
@@ -138,6 +142,15 @@ def _ptr_array(ptrs):
     for i, p in enumerate(ptrs):
         arr[i] = p
     return arr
+
+
+def _pair_table(t, pairs):
+    """Pointers of t[r, l] for pair i = r * layers + l of a contiguous
+    [R, layers, ...] tensor."""
+    if not t.is_contiguous():
+        raise ValueError("tensors must be contiguous")
+    base, stride = t.data_ptr(), t[0, 0].numel() * t.element_size()
+    return _ptr_array([base + stride * i for i in range(pairs)])
 
 
 class Context:
@@ -193,13 +206,7 @@ class Context:
         for t in (qwin, k, v, k_out, v_out, idx_out):
             if not t.is_contiguous():
                 raise ValueError("tensors must be contiguous")
-        pairs = R * Ly
-
-        def table(t):  # pair i = request * layers + layer
-            base, stride = t.data_ptr(), t[0, 0].numel() * t.element_size()
-            return _ptr_array([base + stride * i for i in range(pairs)])
-
-        tq, tk, tv, tko, tvo = (table(t) for t in (qwin, k, v, k_out, v_out))
+        tq, tk, tv, tko, tvo = (_pair_table(t, R * Ly) for t in (qwin, k, v, k_out, v_out))
         _check(load().bacon_compress_all_layers(self.handle, R, tq, tk, tv, N, budget, tko, tvo,
                                                 idx_out.data_ptr(), _stream_ptr(stream)))
         self._last_units, self._last_N = R * Ly * self.kv_heads, N
@@ -230,6 +237,24 @@ class Context:
         self._last_units, self._last_N = R * Ly * self.kv_heads, N
         return ko, vo, ix
 
+    def compress_with_lse(self, qwin, k, v, lse, budget, k_out=None, v_out=None, idx_out=None,
+                          stream=None):
+        """As compress_all_layers, with the window rows' natural-log softmax
+        normalisers lse [R, layers, Hq, W] (fp32, cuda) from the prefill."""
+        R, Ly, Hq, W, d = qwin.shape
+        N = k.shape[3]
+        kept = min(budget, N)
+        shape_o = (R, Ly, self.kv_heads, kept, d)
+        k_out = torch.empty(shape_o, dtype=k.dtype, device=k.device) if k_out is None else k_out
+        v_out = torch.empty(shape_o, dtype=v.dtype, device=v.device) if v_out is None else v_out
+        if idx_out is None:
+            idx_out = torch.empty(shape_o[:-1], dtype=torch.int32, device=k.device)
+        tq, tk, tv, tl, tko, tvo = (_pair_table(t, R * Ly) for t in (qwin, k, v, lse, k_out, v_out))
+        _check(load().bacon_compress_with_lse(self.handle, R, tq, tk, tv, tl, N, budget, tko, tvo,
+                                              idx_out.data_ptr(), _stream_ptr(stream)))
+        self._last_units, self._last_N = R * Ly * self.kv_heads, N
+        return k_out, v_out, idx_out
+
     def compress_adaptive(self, qwin, k, v, budget, alpha=0.2, stream=None):
         """AdaKV-style head budgets.  Returns (k_out, v_out, idx, counts):
         k_out/v_out [R, layers, Hkv * kept, d] and idx [R, layers, Hkv * kept]
@@ -241,9 +266,7 @@ class Context:
         vo = torch.empty_like(ko)
         ix = torch.empty((R, Ly, self.kv_heads * kept), dtype=torch.int32, device=k.device)
         counts = torch.empty((R, Ly, self.kv_heads), dtype=torch.int32, device=k.device)
-        pairs = [(r, l) for r in range(R) for l in range(Ly)]
-        tq, tk, tv, tko, tvo, tix = (_ptr_array([t[r, l].data_ptr() for r, l in pairs])
-                                     for t in (qwin, k, v, ko, vo, ix))
+        tq, tk, tv, tko, tvo, tix = (_pair_table(t, R * Ly) for t in (qwin, k, v, ko, vo, ix))
         _check(load().bacon_compress_adaptive(self.handle, R, tq, tk, tv, N, budget,
                                               float(alpha), tko, tvo, tix, counts.data_ptr(),
                                               _stream_ptr(stream)))

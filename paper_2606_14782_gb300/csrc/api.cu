@@ -294,7 +294,8 @@ bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const vo
                              const void* const* v, int N, const int* layer_budget,
                              void* const* ko, void* const* vo, int32_t* const* idx,
                              cudaStream_t st, bool adaptive = false, int guaranteed = 0,
-                             int32_t* counts = nullptr, size_t unit0 = 0)
+                             int32_t* counts = nullptr, size_t unit0 = 0,
+                             const float* const* prefill_lse = nullptr)
 {
     const int pairs = R * c->layers;
     const Shape s = shape_of(c, c->layers, R, N);
@@ -328,9 +329,17 @@ bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const vo
     const TcArgs ta = tc_args(s, c->d_maps, c->d_maps + kMaxPairs, partial, lse2, B, Q, E, c->err);
     StageEvents prof(c, st);
     prof.mark(0);
-    BACON_CUDA(launch_window_stats_tc(ta, st), "window_stats launch");
-    prof.mark(1);
-    BACON_CUDA(launch_window_combine(s, ta.chunks, partial, lse2, st), "window_combine launch");
+    if (prefill_lse) {
+        // the row normalisers come from the caller's prefill: no pass 1
+        prof.mark(1);
+        LseTable t;
+        for (int i = 0; i < pairs; ++i) t.lse[i] = prefill_lse[i];
+        BACON_CUDA(launch_lse_from_prefill(s, t, lse2, st), "normaliser conversion launch");
+    } else {
+        BACON_CUDA(launch_window_stats_tc(ta, st), "window_stats launch");
+        prof.mark(1);
+        BACON_CUDA(launch_window_combine(s, ta.chunks, partial, lse2, st), "window_combine launch");
+    }
     prof.mark(2);
     BACON_CUDA(launch_window_scores_tc(ta, st), "window_scores launch");
     prof.mark(3);
@@ -722,6 +731,34 @@ bacon_status bacon_compress_layer_budgets(bacon_ctx* ctx, int requests, const vo
     DeviceGuard dg(ctx->device);
     return compress_device(ctx, requests, q_win, k, v, seq_len, layer_budgets, k_out, v_out,
                            idx_out, static_cast<cudaStream_t>(stream));
+}
+
+bacon_status bacon_compress_with_lse(bacon_ctx* ctx, int requests, const void* const* q_win,
+                                     const void* const* k, const void* const* v,
+                                     const float* const* lse, int seq_len, int budget,
+                                     void* const* k_out, void* const* v_out, int32_t* idx_out,
+                                     bacon_stream stream)
+{
+    g_last_error.clear();
+    if (!ctx) return fail(BACON_EINVAL, "null context");
+    if (requests < 1 || requests > ctx->p.max_requests)
+        return fail(BACON_EINVAL, "requests %d outside [1, %d]", requests, ctx->p.max_requests);
+    bacon_status rc = check_seq(ctx, seq_len, budget);
+    if (rc != BACON_OK) return rc;
+    rc = check_pointer_arrays(ctx, requests * ctx->layers, q_win, k, v, k_out, v_out);
+    if (rc != BACON_OK) return rc;
+    if (!lse) return fail(BACON_EINVAL, "null normaliser array");
+    for (int i = 0; i < requests * ctx->layers; ++i)
+        if (!lse[i] || (reinterpret_cast<uintptr_t>(lse[i]) & 3u))
+            return fail(BACON_EINVAL, "normaliser pointer of pair %d must be a 4-byte aligned device pointer", i);
+    if (!idx_out || !aligned16(idx_out)) return fail(BACON_EINVAL, "idx_out must be a 16-byte aligned device pointer");
+    DeviceGuard dg(ctx->device);
+    const int kept = budget < seq_len ? budget : seq_len;
+    std::vector<int> budgets(ctx->layers, budget);
+    int32_t* idx_pairs[kMaxPairs];
+    for (int i = 0; i < requests * ctx->layers; ++i) idx_pairs[i] = idx_out + (size_t)i * ctx->hkv * kept;
+    return compress_device(ctx, requests, q_win, k, v, seq_len, budgets.data(), k_out, v_out,
+                           idx_pairs, static_cast<cudaStream_t>(stream), false, 0, nullptr, 0, lse);
 }
 
 bacon_status bacon_compress_adaptive(bacon_ctx* ctx, int requests, const void* const* q_win,

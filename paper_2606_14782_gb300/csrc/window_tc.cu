@@ -553,6 +553,19 @@ __global__ void window_combine_kernel(Shape s, int chunks, const float2* __restr
     }
 }
 
+// Row normalisers supplied by the caller's prefill attention: per (request,
+// layer) the natural-log LSE of each window row over the keys it sees,
+// [Hq][W] = [Hkv][G W] -> lse2 = LSE log2(e) + log2(G W).
+__global__ void lse_from_prefill_kernel(Shape s, LseTable t, float* __restrict__ lse2)
+{
+    const int u = blockIdx.x;
+    const int pair = u / s.hkv, h = u - pair * s.hkv;
+    const float log2_gw = log2f((float)s.rows);
+    const float* src = t.lse[pair] + (size_t)h * s.rows;
+    for (int r = threadIdx.x; r < s.rows; r += blockDim.x)
+        lse2[(size_t)u * s.rows + r] = fmaf(src[r], kLog2e, log2_gw);
+}
+
 // --------------------------------------------------------------- kernels
 
 template <int D, int PASS>
@@ -656,6 +669,13 @@ cudaError_t launch_impl(const TcArgs& a, cudaStream_t st)
 }  // namespace
 
 int window_tc_max_rows() { return 512; }
+
+cudaError_t launch_lse_from_prefill(const Shape& s, const LseTable& t, float* lse2, cudaStream_t st)
+{
+    const int threads = s.rows < 512 ? ((s.rows + 31) / 32) * 32 : 512;
+    lse_from_prefill_kernel<<<s.units, threads, 0, st>>>(s, t, lse2);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_window_combine(const Shape& s, int chunks, const float2* partial,
                                   float* lse2, cudaStream_t st)

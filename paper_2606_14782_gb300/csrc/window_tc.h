@@ -34,6 +34,14 @@ cudaError_t launch_window_scores_tc(const TcArgs& a, cudaStream_t st);
 cudaError_t launch_window_combine(const Shape& s, int chunks, const float2* partial, float* lse2,
                                   cudaStream_t st);
 
+// Per (request, layer) natural-log softmax normalisers of the window rows,
+// [Hq][W] fp32, as a prefill attention kernel produces them.
+struct LseTable {
+    const float* lse[kMaxPairs];
+};
+cudaError_t launch_lse_from_prefill(const Shape& s, const LseTable& t, float* lse2,
+                                    cudaStream_t st);
+
 // 2-D tensor map over `rows` rows of d bf16 values at `base`: boxes of
 // 64 columns x box_rows rows, 128-byte swizzle, zero fill out of bounds.
 bool encode_rows_map(CUtensorMap* out, const void* base, int d, long long rows, int box_rows);

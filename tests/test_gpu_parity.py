@@ -429,3 +429,52 @@ def test_adaptive_alpha_one_equals_uniform():
     assert (counts.cpu().numpy() == 64).all()
     assert np.array_equal(ix.cpu().numpy().reshape(whole["idx"].shape), whole["idx"])
     assert torch.equal(ko.cpu().reshape(whole["Kc"].shape), whole["Kc"])
+
+
+# --------------------------------------- normalisers supplied by the prefill
+
+def prefill_lse(wl, x):
+    """ln sum_{i <= pos} exp(q . k_i / sqrt(d)) per window row, fp32 on the
+    GPU, as the model's prefill attention would leave it [R, L, Hq, W]."""
+    R, Ly, Hq, W, d = x.qwin.shape
+    H, N, G = wl.kv_heads, wl.seq_len, wl.group
+    out = torch.empty((R, Ly, Hq, W), dtype=torch.float32, device=x.qwin.device)
+    pos = torch.arange(N, device=x.qwin.device)
+    vis = pos[None, :] <= (N - W + torch.arange(W, device=x.qwin.device))[:, None]
+    for r in range(R):
+        for l in range(Ly):
+            q = x.qwin[r, l].float().view(H, G, W, d)
+            k = x.k[r, l].float()
+            s = torch.einsum("hgwd,hnd->hgwn", q, k) / (d ** 0.5)
+            s = s.masked_fill(~vis, float("-inf"))
+            out[r, l] = torch.logsumexp(s, dim=-1).reshape(Hq, W)
+    return out
+
+
+@pytest.mark.parametrize("name,over,budget", [("tiny", {}, 64),
+                                              ("gui", dict(requests=1, layers=3), 1024),
+                                              ("qwen-img", dict(layers=4), 256)])
+def test_prefill_normalisers_path(name, over, budget):
+    wl = workloads.CONFIGS[name].with_(**over)
+    x = workloads.generate(wl, seed=11, device="cuda")
+    lse = prefill_lse(wl, x)
+    full = run_gpu(wl, x, budget)
+    p = bacon.default_params(keep_scores=1, max_seq_len=wl.seq_len, max_requests=wl.requests)
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool,
+                        budget, params=p)
+    ko, vo, idx = ctx.compress_with_lse(x.qwin, x.k, x.v, lse, budget)
+    ctx.sync()
+    shp = (wl.requests, wl.layers, wl.kv_heads, wl.seq_len)
+    got = {k: ctx.scores(k).cpu().numpy().reshape(shp) for k in ("B", "Q", "S")}
+    ctx.close()
+    for k in ("B", "Q", "S"):
+        check_scores(f"{name} {k}", got[k], full[k])
+    if name == "tiny":
+        orc = oracle_run(wl, x, budget)
+        gpu = dict(full, idx=idx.cpu().numpy(), Kc=ko.cpu(), Vc=vo.cpu())
+        for k in ("B", "Q", "S"):
+            gpu[k] = got[k]
+        compare(wl, x, budget, gpu, orc)
+    else:
+        same = (idx.cpu().numpy() == full["idx"]).mean()
+        assert same > 0.99, same
