@@ -363,6 +363,27 @@ def main():
                 "prefill attention, so the first pass over K is skipped"}
     del lse
 
+    # the paper's ablation / sensitivity grid, every variant selected from
+    # one set of window passes (indices only, no gather)
+    variants = list(workloads.SWEEP_VARIANTS)
+    sidx, slam = ctx.sweep(x.qwin, x.k, budget, variants)
+    for _ in range(3):
+        ctx.sweep(x.qwin, x.k, budget, variants, sidx, slam)
+    torch.cuda.synchronize()
+    g0.record(stream)
+    for _ in range(args.steps):
+        ctx.sweep(x.qwin, x.k, budget, variants, sidx, slam)
+    g1.record(stream)
+    torch.cuda.synchronize()
+    sweep_ms = g0.elapsed_time(g1) / args.steps
+    line["ablation_sweep"] = {
+        "variants": len(variants), "ms_per_sweep": sweep_ms,
+        "ms_per_variant": sweep_ms / len(variants),
+        "separate_whole_steps_ms": len(variants) * ms,
+        "what": "bacon_sweep over the component ablation and the m / r sensitivity grid: "
+                "one set of window passes, then calibration and selection per variant"}
+    del sidx, slam
+
     # end to end through the host-buffer C call: H2D inputs, compress, D2H outputs
     if not args.no_e2e:
         del x

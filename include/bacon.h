@@ -200,6 +200,40 @@ bacon_status bacon_compress_adaptive(bacon_ctx* ctx, int requests, const void* c
                                      void* const* v_out, int32_t* const* idx_out,
                                      int32_t* counts_out, bacon_stream stream);
 
+/* Ablation / sensitivity sweep (Sec. 5's component ablation of E, L and T
+ * and its sensitivity study over m and r): every unit is scored under
+ * several hyper-parameter sets while the window passes (Eqs. 1-4, the
+ * dominant cost) run once.  Each variant overrides these fields of the
+ * context's parameters; eps, keep_window and the pool width stay the
+ * context's. */
+#define BACON_MAX_VARIANTS 32
+typedef struct {
+    int r;           /* coherence radius (Eqs. 5-7), >= 0              */
+    int m;           /* persistence depth (Eqs. 8-9), >= 0; 0 = no T  */
+    int rho;         /* scale-matching expansion (Eq. 12), >= 0        */
+    float gamma;     /* calibration strength (Eq. 14), finite, >= 0    */
+    int use_E;       /* terms of Eq. 10 (0 = ablated)                  */
+    int use_L;
+    int use_T;
+} bacon_variant;
+
+/* Selection (Eq. 17) of every (request, layer, kv-head) under each of
+ * n_variants variants (1 <= n_variants <= BACON_MAX_VARIANTS, HOST array),
+ * from one set of window passes.  q_win and k as in
+ * bacon_compress_all_layers; no K/V is gathered.  idx_out is one device
+ * array int32 [n_variants][requests][layers][Hkv][kept], kept =
+ * min(budget, seq_len), each variant's block laid out as that call's;
+ * lambda_out, if not NULL, a device array fp32
+ * [n_variants][requests][layers][Hkv] receiving Eq. 15's lambda.  Variant j
+ * gives the indices bacon_compress_all_layers gives with its fields in the
+ * context's parameters.  Afterwards bacon_get_scores reports BACON_ESTATE
+ * until the next whole-step call.  EINVAL for a variant field out of range;
+ * other errors as bacon_compress_all_layers. */
+bacon_status bacon_sweep(bacon_ctx* ctx, int requests, const void* const* q_win,
+                         const void* const* k, int seq_len, int budget, int n_variants,
+                         const bacon_variant* variants, int32_t* idx_out, float* lambda_out,
+                         bacon_stream stream);
+
 /* Pyramid budget schedule over `layers` layers averaging `budget` (window
  * included): with K = budget - window, K_min = floor(K / beta) and
  * K_max = 2 K - K_min, layer l keeps W + K_min +

@@ -358,3 +358,19 @@ def compress(qwin_bits, k_bits, v_bits, budget, params: Params | None = None,
                 e["Kc"] = gather(k_bits[r, l, h], kept[h])
                 e["Vc"] = gather(v_bits[r, l, h], kept[h])
     return out
+
+
+def sweep(qwin_bits, k_bits, v_bits, budget, variants, params: Params | None = None,
+          threads: int | None = None, units=None, keep_scores=False):
+    """Ablation / sensitivity sweep (Sec. 5.3): the whole step once per
+    variant, a dict of Params fields that override ``params``.  Returns the
+    ``compress`` results in variant order."""
+    params = params or Params()
+    out = []
+    for var in variants:
+        fields = {f: (bool(x) if f.startswith("use_") else x) for f, x in var.items()}
+        out.append(compress(qwin_bits, k_bits, v_bits, budget,
+                            dataclasses.replace(params, **fields), threads, units,
+                            keep_scores=keep_scores))
+    return out
+

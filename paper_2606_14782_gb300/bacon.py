@@ -28,7 +28,9 @@ EXPORTS = ("bacon_default_params", "bacon_init", "bacon_destroy", "bacon_last_er
            "bacon_compress_all_layers", "bacon_compress_host", "bacon_get_scores",
            "bacon_profile_enable", "bacon_profile_read", "bacon_window_scores_noalloc",
            "bacon_compress_layer_budgets", "bacon_pyramid_budgets",
-           "bacon_compress_adaptive", "bacon_compress_with_lse", "bacon_sync")
+           "bacon_compress_adaptive", "bacon_compress_with_lse", "bacon_sweep",
+           "bacon_sync")
+MAX_VARIANTS = 32
 PROFILE_STAGES = ("window_stats", "window_combine", "window_scores", "calibrate_select",
                   "gather")
 
@@ -46,6 +48,13 @@ class Params(ctypes.Structure):
                 ("use_E", ctypes.c_int), ("use_L", ctypes.c_int), ("use_T", ctypes.c_int),
                 ("keep_window", ctypes.c_int), ("max_seq_len", ctypes.c_int),
                 ("max_requests", ctypes.c_int), ("keep_scores", ctypes.c_int)]
+
+
+class Variant(ctypes.Structure):
+    """Mirror of ``bacon_variant``."""
+    _fields_ = [("r", ctypes.c_int), ("m", ctypes.c_int), ("rho", ctypes.c_int),
+                ("gamma", ctypes.c_float), ("use_E", ctypes.c_int), ("use_L", ctypes.c_int),
+                ("use_T", ctypes.c_int)]
 
 
 _lib = None
@@ -95,13 +104,15 @@ def load() -> ctypes.CDLL:
                                             ctypes.POINTER(_vp), _int, _int, ctypes.c_float,
                                             ctypes.POINTER(_vp), ctypes.POINTER(_vp),
                                             ctypes.POINTER(_vp), _vp, _vp]
+    lib.bacon_sweep.argtypes = [_vp, _int, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _int, _int,
+                                _int, ctypes.POINTER(Variant), _vp, _vp, _vp]
     lib.bacon_pyramid_budgets.restype = None
     lib.bacon_window_scores_noalloc.argtypes = [_int, _int, _int, _int, _vp, _vp, _int, _vp,
                                                 _vp, _vp, _vp]
     lib.bacon_profile_enable.argtypes = [_vp, _int]
     lib.bacon_profile_read.argtypes = [_vp, ctypes.POINTER(ctypes.c_double),
                                        ctypes.POINTER(_int), _int]
-    for name in ("bacon_compress_with_lse", "bacon_compress_adaptive",
+    for name in ("bacon_sweep", "bacon_compress_with_lse", "bacon_compress_adaptive",
                  "bacon_compress_layer_budgets",
                  "bacon_window_scores_noalloc",
                  "bacon_profile_enable", "bacon_profile_read",
@@ -272,6 +283,32 @@ class Context:
                                               _stream_ptr(stream)))
         self._last_units, self._last_N = R * Ly * self.kv_heads, N
         return ko, vo, ix, counts
+
+    def sweep(self, qwin, k, budget, variants, idx_out=None, lambda_out=None, stream=None):
+        """Selections under several hyper-parameter sets from one set of
+        window passes.  variants: sequence of dicts with any of r, m, rho,
+        gamma, use_E, use_L, use_T (the rest from the context's parameters).
+        Returns (idx [V, R, layers, Hkv, kept] int32, lambda [V, R, layers,
+        Hkv] fp32)."""
+        R, Ly, Hq, W, d = qwin.shape
+        N = k.shape[3]
+        kept = min(budget, N)
+        nv = len(variants)
+        arr = (Variant * max(nv, 1))()
+        for j, x in enumerate(variants):
+            for f, _ in Variant._fields_:
+                setattr(arr[j], f, x.get(f, getattr(self.params, f)))
+        if idx_out is None:
+            idx_out = torch.empty((nv, R, Ly, self.kv_heads, kept), dtype=torch.int32,
+                                  device=k.device)
+        if lambda_out is None:
+            lambda_out = torch.empty((nv, R, Ly, self.kv_heads), dtype=torch.float32,
+                                     device=k.device)
+        tq, tk = (_pair_table(t, R * Ly) for t in (qwin, k))
+        _check(load().bacon_sweep(self.handle, R, tq, tk, N, budget, nv, arr,
+                                  idx_out.data_ptr(), lambda_out.data_ptr(),
+                                  _stream_ptr(stream)))
+        return idx_out, lambda_out
 
     def compress_host(self, qwin, k, v, budget, k_out=None, v_out=None, idx_out=None,
                       stream=None):

@@ -44,6 +44,7 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 constexpr int kChunkTokens = 1024;  // pass-1 token chunk (multiple of the 128-token tile)
 constexpr int kMaxSeq = 24576;      // calibration keeps 2 x N fp32 in shared memory
+static_assert(kMaxVariants == BACON_MAX_VARIANTS, "variant table size");
 
 // Makes the context's device current for the duration of a call.
 struct DeviceGuard {
@@ -281,8 +282,47 @@ struct StageEvents {
     void commit()
     {
         if (c->prof_on) c->ev_pending.push_back(ev);
+        ev.clear();
+    }
+    ~StageEvents()
+    {
+        for (cudaEvent_t e : ev)  // a call that failed before commit()
+            if (e) c->ev_free.push_back(e);
     }
 };
+
+// Window passes (Eqs. 1-4) of every unit of a call into the scratch slice
+// that starts at unit `unit0`: B, Q and E.  With prefill_lse the window
+// rows' normalisers come from the caller and pass 1 is skipped.
+bacon_status window_passes(bacon_ctx* c, const Shape& s, const void* const* q,
+                           const void* const* k, size_t unit0, const float* const* prefill_lse,
+                           StageEvents& prof, cudaStream_t st)
+{
+    const int pairs = s.units / s.hkv, N = s.N;
+    const int chunks = (N + kTcChunkTokens - 1) / kTcChunkTokens;
+    float* lse2 = c->lse2 + unit0 * c->rows;
+    float2* partial = c->partial + unit0 * chunks * c->rows;
+    bacon_status rc = upload_maps(c, c->d_maps, c->h_maps, c->maps_ev, c->map_key, c->map_key_N,
+                                  kMaxPairs, pairs, q, k, N, st);
+    if (rc != BACON_OK) return rc;
+    const TcArgs ta = tc_args(s, c->d_maps, c->d_maps + kMaxPairs, partial, lse2,
+                              c->B + unit0 * N, c->Q + unit0 * N, c->E + unit0 * N, c->err);
+    prof.mark(0);
+    if (prefill_lse) {
+        prof.mark(1);
+        LseTable t;
+        for (int i = 0; i < pairs; ++i) t.lse[i] = prefill_lse[i];
+        BACON_CUDA(launch_lse_from_prefill(s, t, lse2, st), "normaliser conversion launch");
+    } else {
+        BACON_CUDA(launch_window_stats_tc(ta, st), "window_stats launch");
+        prof.mark(1);
+        BACON_CUDA(launch_window_combine(s, ta.chunks, partial, lse2, st), "window_combine launch");
+    }
+    prof.mark(2);
+    BACON_CUDA(launch_window_scores_tc(ta, st), "window_scores launch");
+    prof.mark(3);
+    return BACON_OK;
+}
 
 // The whole step.  layer_budget[l] is the budget of layer l (window
 // included); idx[pair] receives the pair's [Hkv][min(budget, N)] positions.
@@ -299,15 +339,10 @@ bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const vo
 {
     const int pairs = R * c->layers;
     const Shape s = shape_of(c, c->layers, R, N);
-    // this call's slice of the scratch starts at unit `unit0`
-    const int chunks = (N + kTcChunkTokens - 1) / kTcChunkTokens;
     float* B = c->B + unit0 * N;
-    float* Q = c->Q + unit0 * N;
     float* E = c->E + unit0 * N;
     float* S = c->S + unit0 * N;
     float* lam = c->lam + unit0;
-    float* lse2 = c->lse2 + unit0 * c->rows;
-    float2* partial = c->partial + unit0 * chunks * c->rows;
 
     GatherTable gt;
     CalibArgs a;
@@ -323,26 +358,9 @@ bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const vo
         a.budget[i] = budget;
         a.calib_budget[i] = budget;
     }
-    bacon_status rc = upload_maps(c, c->d_maps, c->h_maps, c->maps_ev, c->map_key, c->map_key_N,
-                                  kMaxPairs, pairs, q, k, N, st);
-    if (rc != BACON_OK) return rc;
-    const TcArgs ta = tc_args(s, c->d_maps, c->d_maps + kMaxPairs, partial, lse2, B, Q, E, c->err);
     StageEvents prof(c, st);
-    prof.mark(0);
-    if (prefill_lse) {
-        // the row normalisers come from the caller's prefill: no pass 1
-        prof.mark(1);
-        LseTable t;
-        for (int i = 0; i < pairs; ++i) t.lse[i] = prefill_lse[i];
-        BACON_CUDA(launch_lse_from_prefill(s, t, lse2, st), "normaliser conversion launch");
-    } else {
-        BACON_CUDA(launch_window_stats_tc(ta, st), "window_stats launch");
-        prof.mark(1);
-        BACON_CUDA(launch_window_combine(s, ta.chunks, partial, lse2, st), "window_combine launch");
-    }
-    prof.mark(2);
-    BACON_CUDA(launch_window_scores_tc(ta, st), "window_scores launch");
-    prof.mark(3);
+    bacon_status rc = window_passes(c, s, q, k, unit0, prefill_lse, prof, st);
+    if (rc != BACON_OK) return rc;
 
     a.B = B;
     a.Ering = E;
@@ -380,6 +398,60 @@ bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const vo
     prof.commit();
     c->last_units = (int)unit0 + s.units;
     c->last_N = N;
+    return BACON_OK;
+}
+
+// Ablation / sensitivity sweep: one set of window passes, then calibration
+// and selection of every unit under each variant.  idx receives int32
+// [variants][pairs][Hkv][kept]; lambda_out (may be null) fp32
+// [variants][units].
+bacon_status sweep_device(bacon_ctx* c, int R, const void* const* q, const void* const* k, int N,
+                          int budget, int variants, const bacon_variant* var, int32_t* idx,
+                          float* lambda_out, cudaStream_t st)
+{
+    const int pairs = R * c->layers;
+    const Shape s = shape_of(c, c->layers, R, N);
+    const int kept = budget < N ? budget : N;
+    CalibArgs a;
+    for (int i = 0; i < pairs; ++i) {
+        a.idx[i] = idx + (size_t)i * c->hkv * kept;
+        a.budget[i] = budget;
+        a.calib_budget[i] = budget;
+    }
+    CalibTable t;
+    for (int j = 0; j < variants; ++j) {
+        Calib& cj = t.c[j];
+        cj = calib_of(c);
+        cj.r = var[j].r;
+        cj.m = var[j].m;
+        cj.rho = var[j].rho;
+        cj.gamma = var[j].gamma;
+        cj.use_E = var[j].use_E;
+        cj.use_L = var[j].use_L;
+        cj.use_T = var[j].use_T;
+    }
+    StageEvents prof(c, st);
+    bacon_status rc = window_passes(c, s, q, k, 0, nullptr, prof, st);
+    if (rc != BACON_OK) return rc;
+    a.B = c->B;
+    a.Ering = c->E;
+    a.ring = c->layers;
+    a.ring_req_stride = (long long)c->layers * c->hkv * N;
+    a.layer0 = 0;
+    a.S = nullptr;
+    a.V = nullptr;
+    a.Bp = nullptr;
+    a.lambda = lambda_out;
+    a.idx_variant_stride = (long long)pairs * c->hkv * kept;
+    a.compute_scores = 1;
+    a.do_select = 1;
+    a.write_S = 0;
+    a.err = c->err;
+    BACON_CUDA(launch_calibrate_sweep(s, t, variants, a, st), "calibrate_sweep launch");
+    prof.mark(4);
+    prof.mark(5);
+    prof.commit();
+    c->last_units = 0;  // S, V, B~ and lambda of the scratch are not this call's
     return BACON_OK;
 }
 
@@ -791,6 +863,40 @@ bacon_status bacon_compress_adaptive(bacon_ctx* ctx, int requests, const void* c
     return compress_device(ctx, requests, q_win, k, v, seq_len, budgets.data(), k_out, v_out,
                            idx_out, static_cast<cudaStream_t>(stream), true, guaranteed,
                            counts_out);
+}
+
+bacon_status bacon_sweep(bacon_ctx* ctx, int requests, const void* const* q_win,
+                         const void* const* k, int seq_len, int budget, int n_variants,
+                         const bacon_variant* variants, int32_t* idx_out, float* lambda_out,
+                         bacon_stream stream)
+{
+    g_last_error.clear();
+    if (!ctx) return fail(BACON_EINVAL, "null context");
+    if (requests < 1 || requests > ctx->p.max_requests)
+        return fail(BACON_EINVAL, "requests %d outside [1, %d]", requests, ctx->p.max_requests);
+    if (n_variants < 1 || n_variants > BACON_MAX_VARIANTS)
+        return fail(BACON_EINVAL, "n_variants %d outside [1, %d]", n_variants, BACON_MAX_VARIANTS);
+    if (!variants) return fail(BACON_EINVAL, "null variant array");
+    for (int j = 0; j < n_variants; ++j) {
+        const bacon_variant& x = variants[j];
+        if (x.r < 0 || x.m < 0 || x.rho < 0)
+            return fail(BACON_EINVAL, "variant %d: r, m, rho must be >= 0", j);
+        if (!(x.gamma >= 0.f) || !(x.gamma < INFINITY))
+            return fail(BACON_EINVAL, "variant %d: gamma must be finite and >= 0", j);
+    }
+    bacon_status rc = check_seq(ctx, seq_len, budget);
+    if (rc != BACON_OK) return rc;
+    const int pairs = requests * ctx->layers;
+    if (!q_win || !k) return fail(BACON_EINVAL, "null pointer array");
+    for (int i = 0; i < pairs; ++i)
+        if (!q_win[i] || !k[i] || !aligned16(q_win[i]) || !aligned16(k[i]))
+            return fail(BACON_EINVAL, "tensor pointer at pair %d is null or not 16-byte aligned", i);
+    if (!idx_out || !aligned16(idx_out)) return fail(BACON_EINVAL, "idx_out must be a 16-byte aligned device pointer");
+    if (lambda_out && (reinterpret_cast<uintptr_t>(lambda_out) & 3u))
+        return fail(BACON_EINVAL, "lambda_out must be 4-byte aligned");
+    DeviceGuard dg(ctx->device);
+    return sweep_device(ctx, requests, q_win, k, seq_len, budget, n_variants, variants, idx_out,
+                        lambda_out, static_cast<cudaStream_t>(stream));
 }
 
 void bacon_pyramid_budgets(int layers, int window, int budget, int beta, int* out)

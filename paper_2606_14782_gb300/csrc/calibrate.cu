@@ -59,8 +59,10 @@ __device__ __forceinline__ void stage(float* dst, const float* src, int n)
     }
 }
 
-__global__ void __launch_bounds__(kThreads)
-calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
+// One unit (request, layer, kv-head) u under hyper-parameters c.  lam_out
+// (may be null) receives lambda; idx_pair is the pair's [Hkv][kept] output.
+__device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, const CalibArgs& a,
+                                               int u, float* lam_out, int32_t* idx_pair)
 {
     extern __shared__ __align__(16) float sm[];
     const int N = s.N, W = s.W;
@@ -72,7 +74,6 @@ calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
     __shared__ float red[33];
     __shared__ int total_s;
 
-    const int u = blockIdx.x;
     const int pair = u / s.hkv, h = u - pair * s.hkv;
     const int rq = pair / s.layers;
     const int layer = a.layer0 + (pair - rq * s.layers);
@@ -185,7 +186,7 @@ calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
             const float stdv = sqrtf(block_sum(vv, red) / (float)M);
             lam = c.gamma * stdb / (stdv + c.eps);
         }
-        if (threadIdx.x == 0) a.lambda[u] = lam;
+        if (threadIdx.x == 0 && lam_out) *lam_out = lam;
         for (int i = threadIdx.x; i < n_cand; i += blockDim.x) Sb[i] = fmaf(lam, Vs[i], Sb[i]);
         __syncthreads();
         if (a.write_S)
@@ -196,7 +197,7 @@ calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
     }
 
     if (!a.do_select) return;
-    int32_t* out = a.idx[pair] + (size_t)h * kept_total;
+    int32_t* out = idx_pair + (size_t)h * kept_total;
     if (keep >= n_cand) {
         for (int i = threadIdx.x; i < n_cand; i += blockDim.x) out[i] = i;
     } else if (keep > 0) {
@@ -219,6 +220,25 @@ calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
     for (int w = threadIdx.x; w < win; w += blockDim.x) out[keep + w] = N - W + w;
 }
 
+__global__ void __launch_bounds__(kThreads)
+calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
+{
+    const int u = blockIdx.x;
+    calibrate_unit(s, c, a, u, a.lambda + u, a.idx[u / s.hkv]);
+}
+
+// Several hyper-parameter sets over the same B and residuals: CTA (u, v)
+// runs unit u under variant v; variant v's indices start v *
+// idx_variant_stride elements after the single-variant layout and its
+// lambdas v * units after a.lambda.
+__global__ void __launch_bounds__(kThreads)
+calibrate_sweep_kernel(Shape s, CalibTable t, CalibArgs a)
+{
+    const int u = blockIdx.x, v = blockIdx.y;
+    float* lam = a.lambda ? a.lambda + (size_t)v * s.units + u : nullptr;
+    calibrate_unit(s, t.c[v], a, u, lam, a.idx[u / s.hkv] + (size_t)v * a.idx_variant_stride);
+}
+
 }  // namespace
 
 size_t calibrate_smem(int N) { return (size_t)2 * N * sizeof(float); }
@@ -231,6 +251,17 @@ cudaError_t launch_calibrate_select(const Shape& s, const Calib& c, const CalibA
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
     calibrate_select_kernel<<<s.units, kThreads, sm, st>>>(s, c, a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_calibrate_sweep(const Shape& s, const CalibTable& t, int variants,
+                                   const CalibArgs& a, cudaStream_t st)
+{
+    const size_t sm = calibrate_smem(s.N);
+    cudaError_t e = cudaFuncSetAttribute(calibrate_sweep_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    calibrate_sweep_kernel<<<dim3(s.units, variants), kThreads, sm, st>>>(s, t, a);
     return cudaGetLastError();
 }
 

@@ -81,6 +81,7 @@ struct CalibArgs {
     int32_t* idx[kMaxPairs];     // per (request, layer): [Hkv][kept] (written when do_select)
     int budget[kMaxPairs];       // kept tokens per head (window included)
     int calib_budget[kMaxPairs]; // budget that sets K in Eq. 12
+    long long idx_variant_stride = 0;  // sweep only: elements between variants' indices
     int compute_scores;  // 1: V, B~, lambda, S from B and the residuals
     int do_select;       // 1: top-B selection into idx
     int write_S;
@@ -88,6 +89,16 @@ struct CalibArgs {
 };
 cudaError_t launch_calibrate_select(const Shape& s, const Calib& c, const CalibArgs& a,
                                     cudaStream_t st);
+
+// Ablation / sensitivity sweep: every unit under each of `variants`
+// hyper-parameter sets (compute_scores and do_select must be 1, write_S 0,
+// V and Bp null).
+constexpr int kMaxVariants = 32;
+struct CalibTable {
+    Calib c[kMaxVariants];
+};
+cudaError_t launch_calibrate_sweep(const Shape& s, const CalibTable& t, int variants,
+                                   const CalibArgs& a, cudaStream_t st);
 
 // Dynamic shared memory of the calibration kernel for N tokens.
 size_t calibrate_smem(int N);

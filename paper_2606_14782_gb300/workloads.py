@@ -202,3 +202,20 @@ def generate(wl: Workload, seed: int = 0, device="cpu") -> Inputs:
 def bf16_bits(t: torch.Tensor):
     """bf16 tensor -> numpy uint16 bit patterns (host copy)."""
     return t.detach().cpu().contiguous().view(torch.int16).numpy().view("uint16")
+
+
+# Hyper-parameter grid of the paper's ablation study (Sec. 5.3).  The
+# component table switches E, L, T off in turn (all three off is the plain
+# backbone score, all on the full method at m = 4, r = 5); the sensitivity
+# tables take m in {0, 2, 4, 6, 8} at r = 5 and r in {0, 3, 5, 7, 9} at
+# m = 4.  Those tables print for m = 0 the scores of the no-T row and for
+# r = 0 those of the no-L row, so m = 0 and r = 0 are taken as those two
+# component variants (by Eq. 6 read literally, r = 0 would give L = E
+# instead).  Each distinct setting is listed once; fields not listed keep
+# the context's values.
+SWEEP_VARIANTS = (
+    [dict(use_E=e, use_L=l, use_T=t, m=4, r=5)
+     for e, l, t in ((1, 1, 1), (0, 0, 0), (1, 0, 1), (1, 1, 0), (0, 1, 1))]
+    + [dict(m=m, r=5) for m in (2, 6, 8)]
+    + [dict(m=4, r=r) for r in (3, 7, 9)]
+)

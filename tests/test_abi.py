@@ -97,3 +97,37 @@ def test_product_path_fails_loudly_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(bacon, "_lib", None)
     with pytest.raises(RuntimeError, match="missing"):
         bacon.load()
+
+
+def test_struct_layouts_match_the_header(tmp_path):
+    """ctypes mirrors of bacon_params and bacon_variant against the C layout."""
+    import os
+    import subprocess
+    src = tmp_path / "layout.c"
+    src.write_text(
+        '#include <stdio.h>\n#include <stddef.h>\n#include "bacon.h"\n'
+        "#define F(T, f) printf(#T \" \" #f \" %zu\\n\", offsetof(T, f));\n"
+        "int main(void) {\n"
+        '  printf("bacon_params size %zu\\n", sizeof(bacon_params));\n'
+        '  printf("bacon_variant size %zu\\n", sizeof(bacon_variant));\n'
+        + "".join(f"  F(bacon_params, {f})\n" for f, _ in bacon.Params._fields_)
+        + "".join(f"  F(bacon_variant, {f})\n" for f, _ in bacon.Variant._fields_)
+        + "  return 0;\n}\n")
+    exe = tmp_path / "layout"
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    subprocess.run(["gcc", "-I", inc, str(src), "-o", str(exe)], check=True)
+    got = {}
+    for line in subprocess.run([str(exe)], check=True, capture_output=True,
+                               text=True).stdout.splitlines():
+        t, f, v = line.split()
+        got[(t, f)] = int(v)
+    for t, cls in (("bacon_params", bacon.Params), ("bacon_variant", bacon.Variant)):
+        assert got[(t, "size")] == ctypes.sizeof(cls), t
+        for f, _ in cls._fields_:
+            assert got[(t, f)] == getattr(cls, f).offset, (t, f)
+
+
+def test_sweep_rejects_null_context(lib):
+    arr = (bacon.Variant * 1)()
+    assert lib.bacon_sweep(None, 1, None, None, 640, 64, 1, arr, None, None,
+                           None) == bacon.BACON_EINVAL

@@ -568,3 +568,68 @@ def test_adaptive_invariants(seed):
     left = {(h, i) for h in range(H) for i in range(N - W)} - {(h, int(i)) for h in range(H) for i in cand[h]}
     key = lambda t: (-S[t[0], t[1]], t[0], t[1])
     assert max(key(t) for t in chosen) < min(key(t) for t in left)
+
+
+# ------------------------------------------ ablation / sensitivity sweep
+
+def _sweep_case(seed=5):
+    from paper_2606_14782_gb300 import workloads
+    wl = workloads.CONFIGS["tiny"].with_(layers=5, seq_len=260, visual=(16, 220))
+    x = workloads.generate(wl, seed=seed)
+    return wl, tuple(workloads.bf16_bits(t) for t in (x.qwin, x.k, x.v))
+
+
+def test_sweep_all_terms_off_is_the_backbone_score():
+    # V = 0 when E, L and T are all switched off (Eq. 10), so S = B~ + lambda 0
+    # = B~ (Eq. 16): the same selection as gamma = 0 with every term on.
+    wl, (qb, kb, vb) = _sweep_case()
+    off, g0 = oracle.sweep(qb, kb, vb, 48, [dict(use_E=0, use_L=0, use_T=0), dict(gamma=0.0)],
+                           threads=4)
+    for key in off:
+        assert np.array_equal(off[key]["idx"], g0[key]["idx"]), key
+
+
+def test_sweep_m_zero_is_no_persistence():
+    # P_0(l) is empty for every l (Eq. 8), so T = 0 (Eq. 9) and m = 0 selects
+    # what use_T = 0 selects, with the same lambda.
+    wl, (qb, kb, vb) = _sweep_case()
+    m0, noT = oracle.sweep(qb, kb, vb, 48, [dict(m=0), dict(use_T=0)], threads=4)
+    for key in m0:
+        assert np.array_equal(m0[key]["idx"], noT[key]["idx"]), key
+        assert m0[key]["lambda"] == noT[key]["lambda"]
+
+
+def test_sweep_radius_covering_the_prompt_makes_L_a_constant():
+    # r >= N - 1: every window of Eq. 6 is the whole prompt, L is the constant
+    # mean of E, so V is the no-L evidence shifted by a constant: Std over M
+    # and hence lambda (Eq. 15) are unchanged and S is shifted uniformly.
+    wl, (qb, kb, vb) = _sweep_case()
+    big, noL = oracle.sweep(qb, kb, vb, 48, [dict(r=wl.seq_len), dict(use_L=0)], threads=4)
+    for key in big:
+        assert np.array_equal(big[key]["idx"], noL[key]["idx"]), key
+        assert abs(big[key]["lambda"] - noL[key]["lambda"]) <= 1e-9 * abs(noL[key]["lambda"])
+
+
+def test_sweep_first_layer_ignores_m():
+    # layer 0 has no preceding layer: T = 0 whatever m is (Eq. 8).
+    wl, (qb, kb, vb) = _sweep_case()
+    res = oracle.sweep(qb, kb, vb, 48, [dict(m=m) for m in (0, 1, 4, 8)], threads=4,
+                       units=[(0, 0, h) for h in range(wl.kv_heads)])
+    for key in res[0]:
+        for other in res[1:]:
+            assert np.array_equal(res[0][key]["idx"], other[key]["idx"]), key
+
+
+def test_sweep_variant_grid_is_distinct_and_covers_the_study():
+    from paper_2606_14782_gb300 import workloads
+    full = dict(use_E=1, use_L=1, use_T=1, m=4, r=5)
+    seen = set()
+    for v in workloads.SWEEP_VARIANTS:
+        k = tuple(sorted({**full, **v}.items()))
+        assert k not in seen, v
+        seen.add(k)
+    comps = {(d["use_E"], d["use_L"], d["use_T"]) for d in map(dict, seen)}
+    assert comps == {(1, 1, 1), (0, 0, 0), (1, 0, 1), (1, 1, 0), (0, 1, 1)}
+    ms = {d["m"] for d in map(dict, seen) if d["r"] == 5 and d["use_T"]}
+    rs = {d["r"] for d in map(dict, seen) if d["m"] == 4 and d["use_L"]}
+    assert ms == {2, 4, 6, 8} and rs == {3, 5, 7, 9}
