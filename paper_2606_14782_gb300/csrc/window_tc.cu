@@ -23,6 +23,8 @@
 // Every wait is bounded: on timeout the CTA raises an abort flag, records
 // kErrTimeout in the error word, drains its own copies and MMAs, frees TMEM
 // and returns.
+#include <cuda_bf16.h>
+
 #include "tc.cuh"
 #include "window_tc.h"
 
@@ -41,11 +43,18 @@ constexpr float kLog2e = 1.4426950408889634f;
 
 struct Smem {
     // offsets in bytes from the 1024-aligned dynamic shared memory base
-    uint32_t q, k, tables, xchg, bars;
+    uint32_t q, k, ones, bias, xchg, bars;
     uint32_t q_half;      // bytes of one 64-column half of the window rows
     uint32_t k_stage;     // bytes of one K tile
     uint32_t total;
 };
+
+// Pass 2 adds two 128 x 64 bf16 operands in the same swizzled layout: a
+// constant one for every token (columns 0-2) and, per job j, the row bias
+// -lse2 / c split into three bf16 parts (columns 16 j .. 16 j + 2), so that
+// one extra K = 16 MMA subtracts each row's normaliser inside the
+// accumulator.
+constexpr uint32_t kBiasOperandBytes = 128u * 128u;
 
 template <int D, int PASS>
 __host__ __device__ inline Smem smem_layout(int q_rows, int stages)
@@ -56,10 +65,9 @@ __host__ __device__ inline Smem smem_layout(int q_rows, int stages)
     s.k_stage = (uint32_t)H * kTileTok * 128u;
     s.q = 0;
     s.k = s.q + H * s.q_half;
-    s.tables = s.k + (uint32_t)stages * s.k_stage;
-    // pass 2 only: per-row nl, qw and last visible key
-    s.xchg = s.tables + (PASS == 2 ? (uint32_t)q_rows * 12u : 0u);
-    s.xchg = (s.xchg + 15u) & ~15u;
+    s.ones = s.k + (uint32_t)stages * s.k_stage;
+    s.bias = s.ones + (PASS == 2 ? kBiasOperandBytes : 0u);
+    s.xchg = s.bias + (PASS == 2 ? kBiasOperandBytes : 0u);
     // partials of groups 1.. (pass 1: per row block; pass 2: two tiles) + flags
     s.bars = s.xchg + (kGroups - 1) * (PASS == 1 ? 4u : 2u) * 128u * 8u + 64u;
     s.bars = (s.bars + 7u) & ~7u;
@@ -67,41 +75,40 @@ __host__ __device__ inline Smem smem_layout(int q_rows, int stages)
     return s;
 }
 
+// Barrier block, 8-byte slots from `base` (a shared-memory address):
+// t_full[4], t_empty[4], q_full, q_empty, drain, ep_all, ep_pair[4], the
+// TMEM base word, the abort word, then k_full[stages], k_empty[stages].
 struct Bars {
-    uint64_t* k_full;   // [stages]
-    uint64_t* k_empty;  // [stages]
-    uint64_t* t_full;   // [4]
-    uint64_t* t_empty;  // [4]
-    uint64_t* q_full;
-    uint64_t* q_empty;
-    uint64_t* drain;
-    uint64_t* ep_all;   // all epilogue warps
-    uint64_t* ep_pair;  // [4] the two epilogue warps of a TMEM lane quarter
-    uint32_t* tmem_base;
-    volatile int* abort;
+    uint32_t base;
+    int stages;
+    __device__ __forceinline__ uint32_t t_full(int i) const { return base + 8u * i; }
+    __device__ __forceinline__ uint32_t t_empty(int i) const { return base + 32u + 8u * i; }
+    __device__ __forceinline__ uint32_t q_full() const { return base + 64u; }
+    __device__ __forceinline__ uint32_t q_empty() const { return base + 72u; }
+    __device__ __forceinline__ uint32_t drain() const { return base + 80u; }
+    __device__ __forceinline__ uint32_t ep_all() const { return base + 88u; }
+    // the epilogue warps of one TMEM lane quarter
+    __device__ __forceinline__ uint32_t ep_pair(int q) const { return base + 96u + 8u * q; }
+    __device__ __forceinline__ uint32_t tmem_slot() const { return base + 128u; }
+    __device__ __forceinline__ uint32_t abort() const { return base + 136u; }
+    __device__ __forceinline__ uint32_t k_full(int st) const { return base + 144u + 8u * st; }
+    __device__ __forceinline__ uint32_t k_empty(int st) const
+    {
+        return base + 144u + 8u * (stages + st);
+    }
 };
 
-__device__ inline Bars bars_at(uint8_t* base, int stages)
+__device__ inline Bars bars_at(uint8_t* p, int stages)
 {
     Bars b;
-    uint64_t* p = reinterpret_cast<uint64_t*>(base);
-    b.k_full = p;
-    b.k_empty = p + stages;
-    b.t_full = p + 2 * stages;
-    b.t_empty = p + 2 * stages + 4;
-    b.q_full = p + 2 * stages + 8;
-    b.q_empty = p + 2 * stages + 9;
-    b.drain = p + 2 * stages + 10;
-    b.ep_all = p + 2 * stages + 11;
-    b.ep_pair = p + 2 * stages + 12;
-    b.tmem_base = reinterpret_cast<uint32_t*>(p + 2 * stages + 16);
-    b.abort = reinterpret_cast<volatile int*>(p + 2 * stages + 17);
+    b.base = smem_u32(p);
+    b.stages = stages;
     return b;
 }
 
 // Barrier among epilogue warps built on an mbarrier (one arrival per warp),
 // so that it shares the bounded, abort-aware wait of the pipeline.
-__device__ inline bool warp_barrier(uint64_t* bar, int& phase, volatile int* abort)
+__device__ inline bool warp_barrier(uint32_t bar, int& phase, uint32_t abort)
 {
     __syncwarp();
     if ((threadIdx.x & 31) == 0) tc::mbar_arrive(bar);
@@ -112,7 +119,7 @@ __device__ inline bool warp_barrier(uint64_t* bar, int& phase, volatile int* abo
 
 __device__ inline void raise_abort(const Bars& b, int* err)
 {
-    *b.abort = 1;
+    tc::st_shared_volatile(b.abort(), 1u);
     if (err) atomicExch(err, tc::kErrTimeout);
 }
 
@@ -123,42 +130,77 @@ __device__ inline void chunk_range(int total, int* c0, int* c1)
     *c1 = (int)(((long long)(blockIdx.x + 1) * total) / gridDim.x);
 }
 
-// Jobs of one tile.  Pass 1: n_jobs row blocks of 128 rows.  Pass 2: the
-// window rows, rounded up to 16-row granules, split into n_jobs groups of at
-// most 128 rows as evenly as granules allow.  The job loops are unrolled over
-// the four possible jobs so the sizes stay in registers.
+// Jobs of one tile: the window rows, in 16-row granules, split into n_jobs
+// jobs of at most 128 rows (8 granules) as evenly as granules allow; job j
+// has n(j) rows starting at row0(j).  Pass 1 uses whole 128-row blocks
+// (8 granules per job).
 struct JobTable {
     int n_jobs;
-    int n[4];
-    int row0[4];
+    int q, rem;  // granules per job, and how many jobs take one more
+    __device__ __forceinline__ int n(int j) const { return 16 * (q + (j < rem ? 1 : 0)); }
+    __device__ __forceinline__ int row0(int j) const { return 16 * (j * q + min(j, rem)); }
 };
 
 __device__ __forceinline__ JobTable make_jobs(int n_jobs, int granules)
 {
     JobTable jt;
     jt.n_jobs = n_jobs;
-    int r = 0;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        const int nj = granules == 0
-                           ? 128
-                           : 16 * (granules / n_jobs + (j < granules % n_jobs ? 1 : 0));
-        jt.n[j] = j < n_jobs ? nj : 0;
-        jt.row0[j] = r;
-        r += jt.n[j];
-    }
+    jt.q = granules / n_jobs;
+    jt.rem = granules - jt.q * n_jobs;
     return jt;
 }
 
 // --------------------------------------------------- producer (TMA, warp 0)
 
-template <int D>
-__device__ __forceinline__ void produce(const TcArgs& a, const Smem& L, uint8_t* sm, const Bars& b, int stages,
-                        int q_rows)
+// Byte offset of element (row, col) of a 128-row x 64-column bf16 operand in
+// the 128-byte-swizzled K-major layout (8-row atoms of 1024 bytes; the
+// 16-byte chunks of a row are permuted by the row's position in its atom).
+__device__ __forceinline__ uint32_t sw128_offset(int row, int col)
+{
+    return (uint32_t)((row >> 3) * 1024 + (row & 7) * 128 + ((((col * 2) >> 4) ^ (row & 7)) << 4) +
+                      ((col * 2) & 15));
+}
+
+// Pass 2 bias operand of unit u: for job j and its row l (window row
+// row0_j + l), columns 16 j .. 16 j + 2 hold -lse2 / c as three bf16 parts
+// whose sum is the fp32 value to about 2^-24; rows beyond the window rows
+// get a huge negative bias so their exponentials vanish.  Written by the 32
+// lanes of the producer warp; columns 16 j + 3 .. stay zero.
+__device__ __forceinline__ void write_bias(const TcArgs& a, uint8_t* bias, int u, const JobTable& jt,
+                                           float inv_c)
+{
+    const Shape& s = a.s;
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        if (j >= jt.n_jobs) break;
+        for (int l = lane; l < jt.n(j); l += 32) {
+            const int r = jt.row0(j) + l;
+            const float x = r < s.rows ? -a.lse2[(size_t)u * s.rows + r] * inv_c : -1.0e38f;
+            const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+            const float r1 = x - __bfloat162float(hi);
+            const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
+            const __nv_bfloat16 lo = __float2bfloat16_rn(r1 - __bfloat162float(mid));
+            const uint32_t off = sw128_offset(l, 16 * j);
+            *reinterpret_cast<uint32_t*>(bias + off) =
+                (uint32_t)__bfloat16_as_ushort(hi) | ((uint32_t)__bfloat16_as_ushort(mid) << 16);
+            *reinterpret_cast<uint32_t*>(bias + off + 4) = (uint32_t)__bfloat16_as_ushort(lo);
+        }
+    }
+}
+
+// All 32 lanes run the loop; lane 0 issues the copies.  At each new unit the
+// window rows are reloaded once the previous unit's MMAs have released them
+// (pass 2 also rewrites the bias operand, a second arrival on q_full).
+template <int D, int PASS>
+__device__ __forceinline__ void produce(const TcArgs& a, const Smem& L, uint8_t* sm, const Bars& b,
+                                        int stages, int q_rows, const JobTable& jt)
 {
     constexpr int H = D / 64;
     const Shape& s = a.s;
+    const int lane = threadIdx.x & 31;
     const int ntiles = (s.N + kTileTok - 1) / kTileTok;
+    const float inv_c = sqrtf((float)D) / kLog2e;
     int c0, c1;
     chunk_range(a.total_chunks, &c0, &c1);
     int cur_u = -1, qloads = 0, kt = 0;
@@ -167,34 +209,46 @@ __device__ __forceinline__ void produce(const TcArgs& a, const Smem& L, uint8_t*
         const int u = g / a.chunks, ci = g - u * a.chunks;
         const int pair = u / s.hkv, h = u - pair * s.hkv;
         if (u != cur_u) {
-            if (!tc::mbar_wait(b.q_empty, (qloads & 1) ^ 1, b.abort)) { ok = false; break; }
-            tc::mbar_arrive_expect_tx(b.q_full, H * L.q_half);
-            for (int kh = 0; kh < H; ++kh)
-                for (int rb = 0; rb < q_rows / kQBox; ++rb)
-                    tc::tma_load_2d(sm + L.q + kh * L.q_half + rb * kQBox * 128, a.qmaps + pair,
-                                    kh * 64, h * s.rows + rb * kQBox, b.q_full);
+            ok = __all_sync(0xffffffffu, tc::mbar_wait(b.q_empty(), (qloads & 1) ^ 1, b.abort()));
+            if (!ok) break;
+            if (lane == 0) {
+                tc::mbar_arrive_expect_tx(b.q_full(), H * L.q_half);
+                for (int kh = 0; kh < H; ++kh)
+                    for (int rb = 0; rb < q_rows / kQBox; ++rb)
+                        tc::tma_load_2d(sm + L.q + kh * L.q_half + rb * kQBox * 128, a.qmaps + pair,
+                                        kh * 64, h * s.rows + rb * kQBox, b.q_full());
+            }
+            if (PASS == 2) {
+                write_bias(a, sm + L.bias, u, jt, inv_c);
+                tc::fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) tc::mbar_arrive(b.q_full());
+            }
             ++qloads;
             cur_u = u;
         }
-        const int t1 = min(ntiles, (ci + 1) * kTilesPerChunk);
-        for (int t = ci * kTilesPerChunk; t < t1; ++t, ++kt) {
-            const int st = kt % stages, n = kt / stages;
-            if (!tc::mbar_wait(b.k_empty + st, (n & 1) ^ 1, b.abort)) { ok = false; break; }
-            tc::mbar_arrive_expect_tx(b.k_full + st, L.k_stage);
-            for (int kh = 0; kh < H; ++kh)
-                tc::tma_load_2d(sm + L.k + st * L.k_stage + kh * kTileTok * 128, a.kmaps + pair,
-                                kh * 64, h * s.N + t * kTileTok, b.k_full + st);
+        if (lane == 0) {
+            const int t1 = min(ntiles, (ci + 1) * kTilesPerChunk);
+            for (int t = ci * kTilesPerChunk; t < t1; ++t, ++kt) {
+                const int st = kt % stages, n = kt / stages;
+                if (!tc::mbar_wait(b.k_empty(st), (n & 1) ^ 1, b.abort())) { ok = false; break; }
+                tc::mbar_arrive_expect_tx(b.k_full(st), L.k_stage);
+                for (int kh = 0; kh < H; ++kh)
+                    tc::tma_load_2d(sm + L.k + st * L.k_stage + kh * kTileTok * 128, a.kmaps + pair,
+                                    kh * 64, h * s.N + t * kTileTok, b.k_full(st));
+            }
         }
+        ok = __shfl_sync(0xffffffffu, ok, 0);
     }
     if (!ok) raise_abort(b, a.err);
+    if (lane != 0) return;
     // drain: the last load of every stage (and of Q) must have landed before
     // this CTA's shared memory can be released
-    volatile int never = 0;
     for (int st = 0; st < stages && st < kt; ++st) {
         const int last = kt - 1 - ((kt - 1 - st) % stages);
-        tc::mbar_wait(b.k_full + st, (last / stages) & 1, &never);
+        tc::mbar_wait(b.k_full(st), (last / stages) & 1, 0u);
     }
-    if (qloads > 0) tc::mbar_wait(b.q_full, (qloads - 1) & 1, &never);
+    if (qloads > 0) tc::mbar_wait(b.q_full(), (qloads - 1) & 1, 0u);
 }
 
 // ------------------------------------------------------ MMA issuer (warp 1)
@@ -207,7 +261,7 @@ __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* s
 {
     const Shape& s = a.s;
     const int ntiles = (s.N + kTileTok - 1) / kTileTok;
-    const uint32_t tmem = *b.tmem_base;
+    const uint32_t tmem = tc::ld_shared(b.tmem_slot());
     const uint32_t sbase = smem_u32(sm);
     constexpr int NBUF = 4;
     constexpr int BUF_COLS = 128;
@@ -218,8 +272,8 @@ __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* s
     for (int g = c0; g < c1 && ok; ++g) {
         const int u = g / a.chunks, ci = g - u * a.chunks;
         if (u != cur_u) {
-            if (cur_u >= 0) tc::umma_commit(b.q_empty);  // previous unit's MMAs release Q
-            if (!tc::mbar_wait(b.q_full, qwaits & 1, b.abort)) { ok = false; break; }
+            if (cur_u >= 0) tc::umma_commit(b.q_empty());  // previous unit's MMAs release Q
+            if (!tc::mbar_wait(b.q_full(), qwaits & 1, b.abort())) { ok = false; break; }
             tc::fence_after_sync();
             ++qwaits;
             cur_u = u;
@@ -227,7 +281,7 @@ __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* s
         const int t1 = min(ntiles, (ci + 1) * kTilesPerChunk);
         for (int t = ci * kTilesPerChunk; t < t1 && ok; ++t, ++kt) {
             const int st = kt % stages, n = kt / stages;
-            if (!tc::mbar_wait(b.k_full + st, n & 1, b.abort)) { ok = false; break; }
+            if (!tc::mbar_wait(b.k_full(st), n & 1, b.abort())) { ok = false; break; }
             tc::fence_after_sync();
             const uint32_t kaddr = sbase + L.k + st * L.k_stage;
 #pragma unroll
@@ -235,11 +289,14 @@ __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* s
                 if (j >= jt.n_jobs) break;
                 const int buf = job % NBUF, nb = job / NBUF;
                 ++job;
-                if (!tc::mbar_wait(b.t_empty + buf, (nb & 1) ^ 1, b.abort)) { ok = false; break; }
+                if (!tc::mbar_wait(b.t_empty(buf), (nb & 1) ^ 1, b.abort())) { ok = false; break; }
                 tc::fence_after_sync();
                 const uint32_t d_tmem = tmem + buf * BUF_COLS;
-                const uint32_t idesc = tc::idesc_bf16(128, jt.n[j]);
-                const uint32_t qaddr = sbase + L.q + jt.row0[j] * 128;
+                const uint32_t idesc = tc::idesc_bf16(128, jt.n(j));
+                const uint32_t qaddr = sbase + L.q + jt.row0(j) * 128;
+                if (PASS == 2)  // D = -lse2 / c per row (columns of D), then += K Q^T
+                    tc::umma_bf16(d_tmem, tc::sdesc_sw128(sbase + L.ones),
+                                  tc::sdesc_sw128(sbase + L.bias + 32 * j), idesc, 0);
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
                     const int kh = kk / 4;
@@ -249,18 +306,17 @@ __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* s
                     if (PASS == 1)
                         tc::umma_bf16(d_tmem, qd, kd, idesc, kk > 0);
                     else
-                        tc::umma_bf16(d_tmem, kd, qd, idesc, kk > 0);
+                        tc::umma_bf16(d_tmem, kd, qd, idesc, 1);
                 }
-                tc::umma_commit(b.t_full + buf);
+                tc::umma_commit(b.t_full(buf));
             }
-            tc::umma_commit(b.k_empty + st);  // the K stage is free once these MMAs finish
+            tc::umma_commit(b.k_empty(st));  // the K stage is free once these MMAs finish
         }
     }
     if (!ok) raise_abort(b, a.err);
     // every MMA issued must complete before TMEM is released
-    tc::umma_commit(b.drain);
-    volatile int never = 0;
-    tc::mbar_wait(b.drain, 0, &never);
+    tc::umma_commit(b.drain());
+    tc::mbar_wait(b.drain(), 0, 0u);
     (void)q_rows;
 }
 
@@ -278,7 +334,7 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int quarter = warp & 3;        // TMEM lanes this warp may access
     const int group = (warp - 2) >> 2;   // which 32 tokens of each job
-    const uint32_t tmem = *b.tmem_base;
+    const uint32_t tmem = tc::ld_shared(b.tmem_slot());
     float2* xchg = reinterpret_cast<float2*>(sm + L.xchg);  // [group - 1][rb][128]
     const int nrb = q_rows / 128;
     const float c = kLog2e * rsqrtf((float)D);
@@ -307,35 +363,39 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
                 if (rb >= nrb) break;
                 const int buf = job & 3, nb = job >> 2;
                 ++job;
-                if (!tc::mbar_wait(b.t_full + buf, nb & 1, b.abort)) { ok = false; break; }
+                if (!tc::mbar_wait(b.t_full(buf), nb & 1, b.abort())) { ok = false; break; }
                 tc::fence_after_sync();
                 float v[32];
                 tc::tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + buf * 128 + group * 32, v);
                 tc::tmem_ld_wait_regs32(v);
                 tc::fence_before_sync();
                 __syncwarp();
-                if (lane == 0) tc::mbar_arrive(b.t_empty + buf);
+                if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
                 if (need_mask) {
 #pragma unroll
                     for (int j = 0; j < 32; ++j)
                         if (tok0 + j > vis[rb]) v[j] = -INFINITY;
                 }
-                float mx[4];
+                // max of 32 by a tree of 3-input maxima
+                float m9[11];
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    mx[i] = tc::max3(tc::max3(v[8 * i], v[8 * i + 1], v[8 * i + 2]),
-                                     tc::max3(v[8 * i + 3], v[8 * i + 4], v[8 * i + 5]),
-                                     fmaxf(v[8 * i + 6], v[8 * i + 7]));
-                const float m_new = fmaxf(m_run[rb], fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * c);
+                for (int i = 0; i < 10; ++i) m9[i] = tc::max3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+                m9[10] = fmaxf(v[30], v[31]);
+                const float mA = tc::max3(m9[0], m9[1], m9[2]);
+                const float mB = tc::max3(m9[3], m9[4], m9[5]);
+                const float mC = tc::max3(m9[6], m9[7], m9[8]);
+                const float mD = fmaxf(m9[9], m9[10]);
+                const float m_new = fmaxf(m_run[rb], fmaxf(tc::max3(mA, mB, mC), mD) * c);
                 if (m_new != -INFINITY) {
                     const unsigned long long nm2 = tc::pack2(-m_new, -m_new);
-                    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+                    unsigned long long acc[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
                     for (int j = 0; j < 32; j += 2) {
                         const float2 tt = tc::unpack2(tc::fma2(tc::pack2(v[j], v[j + 1]), c2, nm2));
-                        acc[(j >> 1) & 3] += fast_exp2(tt.x) + fast_exp2(tt.y);
+                        acc[(j >> 1) & 3] = tc::add2(acc[(j >> 1) & 3], tc::pack2(fast_exp2(tt.x), fast_exp2(tt.y)));
                     }
-                    z_run[rb] = z_run[rb] * fast_exp2(m_run[rb] - m_new) + ((acc[0] + acc[1]) + (acc[2] + acc[3]));
+                    const float2 s2 = tc::unpack2(tc::add2(tc::add2(acc[0], acc[1]), tc::add2(acc[2], acc[3])));
+                    z_run[rb] = z_run[rb] * fast_exp2(m_run[rb] - m_new) + (s2.x + s2.y);
                     m_run[rb] = m_new;
                 }
             }
@@ -345,7 +405,7 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
         if (group > 0)
             for (int rb = 0; rb < nrb; ++rb)
                 xchg[((group - 1) * 4 + rb) * 128 + quarter * 32 + lane] = make_float2(m_run[rb], z_run[rb]);
-        if (!warp_barrier(b.ep_all, ep_phase, b.abort)) { ok = false; break; }
+        if (!warp_barrier(b.ep_all(), ep_phase, b.abort())) { ok = false; break; }
         if (group == 0) {
             for (int rb = 0; rb < nrb; ++rb) {
                 const int r = rb * 128 + quarter * 32 + lane;
@@ -364,157 +424,166 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
                     a.partial[((size_t)u * a.chunks + ci) * s.rows + r] = make_float2(M, Z);
             }
         }
-        if (!warp_barrier(b.ep_all, ep_phase, b.abort)) { ok = false; break; }
+        if (!warp_barrier(b.ep_all(), ep_phase, b.abort())) { ok = false; break; }
     }
     if (!ok) raise_abort(b, a.err);
 }
 
 // ------------------------------------------------ epilogue, pass 2 (scores)
 
-// Thread = one token (TMEM lane); the 32-column chunks of a tile's jobs are
-// dealt alternately to the two warps of a lane quarter.  Per-row terms in
-// shared memory: nl = -(log2 of the row's softmax normaliser times G W);
-// qw = W on the rows of the last window position (their sum is Q), else 0;
-// the last key position each row may see; and, per 16-row group, whether
-// its last row is a last-position row (with W a multiple of 16 that is the
-// only place such a row can sit: FASTQ).
-struct ScoreTabs {
-    const float* nl;  // [q_rows] nl, then [q_rows] qw, then [q_rows] vis
-    int q_rows;
-    const uint8_t* qflag;
-    __device__ __forceinline__ const float* qw() const { return nl + q_rows; }
-    __device__ __forceinline__ const int* vis() const
-    {
-        return reinterpret_cast<const int*>(nl + 2 * q_rows);
-    }
+// Thread = one token (TMEM lane).  The accumulator of a job already holds
+// logit - lse2 / c for each of its window rows (columns), so a column's share
+// of B is 2^(c D) (= A_{q,i} / (G W)).  Each job's columns are cut into
+// 32-column slices, one per group, rotated from job to job so that the short
+// last slice moves between the groups.  Q sums the columns of last-position
+// rows (scaled by W at the end, so that the G heads' rows average to Q).
+struct ScoreCtx {
+    unsigned long long c2;
+    int N, W;
+    uint32_t qmask;  // bit g: 16-row granule g ends on a last-position row
 };
 
-template <int NV, bool FASTQ, bool MASK>
-__device__ __forceinline__ void score_chunk(const float* v, int r, const ScoreTabs& tb,
-                                            unsigned long long c2, int tok, float* bacc,
-                                            float* qacc, float& qlast)
+template <int NC, bool FASTQ, bool MASK>
+__device__ __forceinline__ void score_slice(float* v, int r0, int tok, const ScoreCtx& k,
+                                            unsigned long long* bacc, float& qacc)
 {
+    if (MASK) {
+        // window row r sits at position N - W + (r mod W) and sees keys up to
+        // it: this token is hidden from the rows with r mod W < tok - (N - W)
+        const int lim = tok - (k.N - k.W);
+        if (FASTQ) {
+            // W % 16 == 0: r mod W runs up by one inside each 16-row granule
 #pragma unroll
-    for (int jj = 0; jj < NV; jj += 4) {
-        const float4 nl = *reinterpret_cast<const float4*>(tb.nl + r + jj);
-        const float2 t0 = tc::unpack2(tc::fma2(tc::pack2(v[jj], v[jj + 1]), c2, tc::pack2(nl.x, nl.y)));
-        const float2 t1 = tc::unpack2(tc::fma2(tc::pack2(v[jj + 2], v[jj + 3]), c2, tc::pack2(nl.z, nl.w)));
-        float x0 = fast_exp2(t0.x), x1 = fast_exp2(t0.y);
-        float x2 = fast_exp2(t1.x), x3 = fast_exp2(t1.y);
-        if (MASK) {
-            const int4 vis = *reinterpret_cast<const int4*>(tb.vis() + r + jj);
-            if (tok > vis.x) x0 = 0.f;
-            if (tok > vis.y) x1 = 0.f;
-            if (tok > vis.z) x2 = 0.f;
-            if (tok > vis.w) x3 = 0.f;
+            for (int g = 0; g < NC / 16; ++g) {
+                const int th = lim - (r0 + 16 * g) % k.W;
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                    if (j < th) v[16 * g + j] = -INFINITY;
+            }
+        } else {
+            int rm = r0 % k.W;
+#pragma unroll
+            for (int j = 0; j < NC; ++j) {
+                if (rm < lim) v[j] = -INFINITY;
+                rm = rm + 1 == k.W ? 0 : rm + 1;
+            }
         }
-        bacc[0] += x0;
-        bacc[1] += x1;
-        bacc[2] += x2;
-        bacc[3] += x3;
-        if (!FASTQ) {
-            const float4 qw = *reinterpret_cast<const float4*>(tb.qw() + r + jj);
-            qacc[0] = fmaf(x0, qw.x, qacc[0]);
-            qacc[1] = fmaf(x1, qw.y, qacc[1]);
-            qacc[0] = fmaf(x2, qw.z, qacc[0]);
-            qacc[1] = fmaf(x3, qw.w, qacc[1]);
-        } else if ((jj & 15) == 12) {
-            if (tb.qflag[(r + jj) >> 4]) qlast += x3;  // the group's last column
+    }
+    int rm = FASTQ ? 0 : r0 % k.W;
+#pragma unroll
+    for (int j = 0; j < NC; j += 2) {
+        const float2 t = tc::unpack2(tc::mul2(tc::pack2(v[j], v[j + 1]), k.c2));
+        const float x0 = fast_exp2(t.x), x1 = fast_exp2(t.y);
+        bacc[(j >> 1) & 1] = tc::add2(bacc[(j >> 1) & 1], tc::pack2(x0, x1));
+        if (FASTQ) {
+            // with W a multiple of 16 only a granule's last row can be a last-position row
+            if ((j & 15) == 14 && ((k.qmask >> ((r0 + j) >> 4)) & 1u)) qacc += x1;
+        } else {
+            if (rm == k.W - 1) qacc += x0;
+            rm = rm + 1 == k.W ? 0 : rm + 1;
+            if (rm == k.W - 1) qacc += x1;
+            rm = rm + 1 == k.W ? 0 : rm + 1;
         }
     }
 }
 
 template <bool FASTQ, bool MASK>
-__device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int group, int quarter,
-                                           uint32_t tmem,
-                                           const Bars& b, const ScoreTabs& tb,
-                                           unsigned long long c2, int tok, float* bacc,
-                                           float* qacc, float& qlast)
+__device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int group, uint32_t tl,
+                                           const Bars& b, const ScoreCtx& k, int tok,
+                                           unsigned long long* bacc, float& qacc)
 {
     const int lane = threadIdx.x & 31;
-    int kglob = 0;  // 16-column piece index of the tile where this job starts
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
         if (j >= jt.n_jobs) break;
         const int buf = job & 3, nb = job >> 2;
+        const int sl = (group + job) & (kGroups - 1);
         ++job;
-        if (!tc::mbar_wait(b.t_full + buf, nb & 1, b.abort)) return false;
+        if (!tc::mbar_wait(b.t_full(buf), nb & 1, b.abort())) return false;
         tc::fence_after_sync();
-        const int np = jt.n[j] / 16, r0 = jt.row0[j];
-        const uint32_t taddr = tmem + ((uint32_t)(quarter * 32) << 16) + buf * 128;
-        // pieces i = group, group + 4, ... of the tile that fall in this job
-        for (int i = (group - kglob) & (kGroups - 1); i < np; i += kGroups) {
+        const int np = jt.n(j) >> 4, ns = (np + 1) >> 1;
+        const uint32_t taddr = tl + buf * 128 + 32 * sl;
+        const int r0 = jt.row0(j) + 32 * sl;
+        const bool mine = sl < ns, two = 2 * sl + 1 < np;
+        if (!MASK) {
+            float v[32];
+            if (mine) {
+                if (two) {
+                    tc::tmem_ld32(taddr, v);
+                    tc::tmem_ld_wait_regs32(v);
+                } else {
+                    tc::tmem_ld16(taddr, v);
+                    tc::tmem_ld_wait_regs16(v);
+                }
+            }
+            tc::fence_before_sync();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
+            if (mine) {
+                if (two)
+                    score_slice<32, FASTQ, false>(v, r0, tok, k, bacc, qacc);
+                else
+                    score_slice<16, FASTQ, false>(v, r0, tok, k, bacc, qacc);
+            }
+        } else {
+            // tiles that reach into the window (one or two per unit) go 16
+            // columns at a time, keeping the masking's register demand low
             float v[16];
-            tc::tmem_ld16(taddr + 16 * i, v);
-            tc::tmem_ld_wait_regs16(v);
-            score_chunk<16, FASTQ, MASK>(v, r0 + 16 * i, tb, c2, tok, bacc, qacc, qlast);
+            for (int h = 0; h < (mine ? (two ? 2 : 1) : 0); ++h) {
+                tc::tmem_ld16(taddr + 16 * h, v);
+                tc::tmem_ld_wait_regs16(v);
+                score_slice<16, FASTQ, true>(v, r0 + 16 * h, tok, k, bacc, qacc);
+            }
+            tc::fence_before_sync();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
         }
-        kglob += np;
-        tc::fence_before_sync();
-        __syncwarp();
-        if (lane == 0) tc::mbar_arrive(b.t_empty + buf);
     }
     return true;
 }
 
 template <int D, bool FASTQ>
-__device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, uint8_t* sm, const Bars& b,
-                                int q_rows, const JobTable& jt)
+__device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, uint8_t* sm,
+                                                const Bars& b, const JobTable& jt)
 {
     const Shape& s = a.s;
     const int ntiles = (s.N + kTileTok - 1) / kTileTok;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int quarter = warp & 3;
     const int group = (warp - 2) >> 2;
-    const int et = threadIdx.x - 64;  // among the epilogue threads
-    const uint32_t tmem = *b.tmem_base;
-    float* nl_s = reinterpret_cast<float*>(sm + L.tables);  // [q_rows]
-    float* qw_s = nl_s + q_rows;                            // [q_rows]
-    int* vis_s = reinterpret_cast<int*>(qw_s + q_rows);     // [q_rows]
-    uint8_t* qflag_s = reinterpret_cast<uint8_t*>(sm + L.xchg) + 2 * (kGroups - 1) * 128 * 8;  // [q_rows / 16]
-    float2* xs = reinterpret_cast<float2*>(sm + L.xchg);    // [2][kGroups - 1][128]
-    const ScoreTabs tb{nl_s, q_rows, qflag_s};
+    const uint32_t tl = tc::ld_shared(b.tmem_slot()) + ((uint32_t)(quarter * 32) << 16);
+    float2* xs = reinterpret_cast<float2*>(sm + L.xchg);  // [2][kGroups - 1][128]
+    ScoreCtx k;
     const float c = kLog2e * rsqrtf((float)D);
-    const unsigned long long c2 = tc::pack2(c, c);
+    k.c2 = tc::pack2(c, c);
+    k.N = s.N;
+    k.W = s.W;
+    k.qmask = 0u;
+    for (int g = 0; g < 32; ++g)
+        if (16 * g + 15 < s.rows && (16 * g + 15) % s.W == s.W - 1) k.qmask |= 1u << g;
     int c0, c1;
     chunk_range(a.total_chunks, &c0, &c1);
-    int cur_u = -1, job = 0, ep_phase = 0, pair_phase = 0;
+    int job = 0, pair_phase = 0;
     bool ok = true;
     for (int g = c0; g < c1 && ok; ++g) {
         const int u = g / a.chunks, ci = g - u * a.chunks;
-        if (u != cur_u) {
-            // all epilogue warps are done with the previous unit's tables
-            if (!warp_barrier(b.ep_all, ep_phase, b.abort)) { ok = false; break; }
-            for (int r = et; r < q_rows; r += kEpiThreads) {
-                const bool real = r < s.rows;
-                const bool last = real && (r % s.W) == s.W - 1;
-                nl_s[r] = real ? -a.lse2[(size_t)u * s.rows + r] : -INFINITY;
-                qw_s[r] = last ? (float)s.W : 0.f;
-                vis_s[r] = s.N - s.W + (r % s.W);
-                if ((r & 15) == 15) qflag_s[r >> 4] = last ? 1 : 0;
-            }
-            if (!warp_barrier(b.ep_all, ep_phase, b.abort)) { ok = false; break; }
-            cur_u = u;
-        }
         const int t1 = min(ntiles, (ci + 1) * kTilesPerChunk);
         for (int t = ci * kTilesPerChunk; t < t1 && ok; ++t) {
             const int tok = t * kTileTok + quarter * 32 + lane;
             const bool need_mask = t * kTileTok + kTileTok - 1 > s.N - s.W;
-            float bacc[4] = {0.f, 0.f, 0.f, 0.f};
-            float qacc[2] = {0.f, 0.f};
-            float qlast = 0.f;
-            ok = need_mask ? score_tile<FASTQ, true>(jt, job, group, quarter, tmem, b, tb, c2, tok,
-                                                     bacc, qacc, qlast)
-                           : score_tile<FASTQ, false>(jt, job, group, quarter, tmem, b, tb, c2, tok,
-                                                      bacc, qacc, qlast);
+            unsigned long long bacc[2] = {0ull, 0ull};
+            float qacc = 0.f;
+            ok = need_mask ? score_tile<FASTQ, true>(jt, job, group, tl, b, k, tok, bacc, qacc)
+                           : score_tile<FASTQ, false>(jt, job, group, tl, b, k, tok, bacc, qacc);
             if (!ok) break;
-            float bsum = (bacc[0] + bacc[1]) + (bacc[2] + bacc[3]);
-            float qsum = FASTQ ? qlast * (float)s.W : qacc[0] + qacc[1];
+            const float2 b2 = tc::unpack2(tc::add2(bacc[0], bacc[1]));
+            float bsum = b2.x + b2.y;
+            float qsum = qacc * (float)s.W;
             // the groups' partial sums of a token meet in shared memory
             // (double-buffered by tile)
             float2* slots = xs + (t & 1) * (kGroups - 1) * 128 + quarter * 32 + lane;
             if (group > 0) slots[(group - 1) * 128] = make_float2(bsum, qsum);
-            if (!warp_barrier(b.ep_pair + quarter, pair_phase, b.abort)) { ok = false; break; }
+            if (!warp_barrier(b.ep_pair(quarter), pair_phase, b.abort())) { ok = false; break; }
             if (group == 0 && tok < s.N) {
                 for (int gg = 0; gg < kGroups - 1; ++gg) {
                     const float2 o = slots[gg * 128];
@@ -582,40 +651,53 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, int q_
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < stages; ++i) {
-            tc::mbar_init(b.k_full + i, 1);
-            tc::mbar_init(b.k_empty + i, 1);
+            tc::mbar_init(b.k_full(i), 1);
+            tc::mbar_init(b.k_empty(i), 1);
         }
         for (int i = 0; i < 4; ++i) {
-            tc::mbar_init(b.t_full + i, 1);
-            tc::mbar_init(b.t_empty + i, kEpiThreads / 32);  // one arrival per epilogue warp
+            tc::mbar_init(b.t_full(i), 1);
+            tc::mbar_init(b.t_empty(i), kEpiThreads / 32);  // one arrival per epilogue warp
         }
-        tc::mbar_init(b.q_full, 1);
-        tc::mbar_init(b.q_empty, 1);
-        tc::mbar_init(b.drain, 1);
-        tc::mbar_init(b.ep_all, kEpiThreads / 32);
-        for (int i = 0; i < 4; ++i) tc::mbar_init(b.ep_pair + i, kGroups);
-        *b.abort = 0;
+        tc::mbar_init(b.q_full(), PASS == 2 ? 2 : 1);  // pass 2: TMA bytes + the bias writes
+        tc::mbar_init(b.q_empty(), 1);
+        tc::mbar_init(b.drain(), 1);
+        tc::mbar_init(b.ep_all(), kEpiThreads / 32);
+        for (int i = 0; i < 4; ++i) tc::mbar_init(b.ep_pair(i), kGroups);
+        tc::st_shared_volatile(b.abort(), 0u);
         tc::fence_barrier_init();
     }
     if (warp == 1) {
-        tc::tmem_alloc(b.tmem_base, kTmemCols);
+        tc::tmem_alloc(b.tmem_slot(), kTmemCols);
         tc::tmem_relinquish();
+    }
+    if (PASS == 2 && threadIdx.x >= 64 && threadIdx.x < 64 + 128) {
+        // constant operand: 1 in columns 0-2 of every token row; the bias
+        // operand starts zeroed (the producer fills columns 16 j .. 16 j + 2)
+        const int row = threadIdx.x - 64;
+        uint4* ones = reinterpret_cast<uint4*>(sm + L.ones + row * 128);
+        uint4* bias = reinterpret_cast<uint4*>(sm + L.bias + row * 128);
+        for (int q = 0; q < 8; ++q) ones[q] = bias[q] = make_uint4(0u, 0u, 0u, 0u);
+        const uint32_t off = sw128_offset(row, 0) - (uint32_t)row * 128u;
+        uint8_t* r = sm + L.ones + row * 128 + off;
+        *reinterpret_cast<uint32_t*>(r) = 0x3F803F80u;  // bf16 1.0, 1.0
+        *reinterpret_cast<uint32_t*>(r + 4) = 0x00003F80u;
+        tc::fence_proxy_async_smem();
     }
     tc::fence_before_sync();
     __syncthreads();
     tc::fence_after_sync();
 
     if (warp == 0) {
-        if (tc::elect_one()) produce<D>(a, L, sm, b, stages, q_rows);
+        produce<D, PASS>(a, L, sm, b, stages, q_rows, jt);
     } else if (warp == 1) {
         if (tc::elect_one()) issue<D, PASS>(a, L, sm, b, stages, q_rows, jt);
     } else {
         if (PASS == 1)
             epilogue_stats<D>(a, L, sm, b, q_rows);
         else if (a.s.W % 16 == 0)
-            epilogue_scores<D, true>(a, L, sm, b, q_rows, jt);
+            epilogue_scores<D, true>(a, L, sm, b, jt);
         else
-            epilogue_scores<D, false>(a, L, sm, b, q_rows, jt);
+            epilogue_scores<D, false>(a, L, sm, b, jt);
     }
 
     tc::fence_before_sync();
@@ -623,7 +705,7 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, int q_
     if (warp == 1) {
         __syncwarp();
         tc::fence_after_sync();
-        tc::tmem_dealloc(*b.tmem_base, kTmemCols);
+        tc::tmem_dealloc(tc::ld_shared(b.tmem_slot()), kTmemCols);
     }
 }
 
@@ -647,7 +729,7 @@ cudaError_t launch_impl(const TcArgs& a, cudaStream_t st)
     const int rows = a.s.rows;
     // pass 1: whole 128-row MMA blocks; pass 2: whole 64-row TMA boxes
     const int q_rows = PASS == 1 ? (rows + 127) / 128 * 128 : (rows + kQBox - 1) / kQBox * kQBox;
-    const int granules = PASS == 1 ? 0 : (rows + 15) / 16;
+    const int granules = PASS == 1 ? q_rows / 16 : (rows + 15) / 16;
     const int n_jobs = PASS == 1 ? q_rows / 128 : (granules + 7) / 8;
     int stages = 4;
     const size_t budget = 227 * 1024 - 1024;
