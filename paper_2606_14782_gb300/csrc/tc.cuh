@@ -206,14 +206,16 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v)
 // Shared-memory matrix descriptor for a K-major operand stored in the
 // 128-byte-swizzled layout TMA writes (rows of 128 bytes, 8-row atoms of
 // 1024 bytes, atoms 1024-byte aligned).
-__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr)
+// `atom_stride` is the byte distance between consecutive 8-row atoms (1024
+// for a dense operand; 0 makes every 8-row group read the same atom).
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t atom_stride = 1024u)
 {
     uint64_t d = 0;
-    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);  // start address
-    d |= (uint64_t)1 << 16;                     // leading byte offset (unused here)
-    d |= (uint64_t)(1024 >> 4) << 32;           // stride byte offset: next 8-row atom
-    d |= (uint64_t)1 << 46;                     // descriptor version for tcgen05
-    d |= (uint64_t)2 << 61;                     // 128-byte swizzle
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);     // start address
+    d |= (uint64_t)1 << 16;                        // leading byte offset (unused here)
+    d |= (uint64_t)((atom_stride >> 4) & 0x3FFFu) << 32;  // stride byte offset
+    d |= (uint64_t)1 << 46;                        // descriptor version for tcgen05
+    d |= (uint64_t)2 << 61;                        // 128-byte swizzle
     return d;
 }
 

@@ -49,15 +49,19 @@ struct Smem {
     uint32_t total;
 };
 
-// Pass 2 adds two 128 x 64 bf16 operands in the same swizzled layout: a
-// constant one for every token (columns 0-2) and, per job j, the row bias
-// -lse2 / c split into three bf16 parts (columns 16 j .. 16 j + 2), so that
-// one extra K = 16 MMA subtracts each row's normaliser inside the
-// accumulator.
+// Pass 2 adds two bf16 operands in the same swizzled layout: a constant one
+// for every token (columns 0-2) and, per job j, the row bias -lse2 / c split
+// into three bf16 parts (columns 16 j .. 16 j + 2), so that one extra
+// K = 16 MMA subtracts each row's normaliser inside the accumulator.  The
+// bias operand has 128 rows x 64 columns.  The constant operand is 128
+// identical rows; when shared memory is short (512 window rows of d = 128)
+// only its first 8-row atom is stored and the descriptor's 8-row stride is
+// zero, so every group of 8 token rows reads the same atom.
 constexpr uint32_t kBiasOperandBytes = 128u * 128u;
+constexpr uint32_t kOnesAtomBytes = 8u * 128u;
 
 template <int D, int PASS>
-__host__ __device__ inline Smem smem_layout(int q_rows, int stages)
+__host__ __device__ inline Smem smem_layout(int q_rows, int stages, bool ones_atom = false)
 {
     Smem s;
     constexpr int H = D / 64;
@@ -66,7 +70,7 @@ __host__ __device__ inline Smem smem_layout(int q_rows, int stages)
     s.q = 0;
     s.k = s.q + H * s.q_half;
     s.ones = s.k + (uint32_t)stages * s.k_stage;
-    s.bias = s.ones + (PASS == 2 ? kBiasOperandBytes : 0u);
+    s.bias = s.ones + (PASS == 2 ? (ones_atom ? kOnesAtomBytes : kBiasOperandBytes) : 0u);
     s.xchg = s.bias + (PASS == 2 ? kBiasOperandBytes : 0u);
     // partials of groups 1.. (pass 1: per row block; pass 2: two tiles) + flags
     s.bars = s.xchg + (kGroups - 1) * (PASS == 1 ? 4u : 2u) * 128u * 8u + 64u;
@@ -257,7 +261,7 @@ __device__ __forceinline__ void produce(const TcArgs& a, const Smem& L, uint8_t*
 // Pass 2: A = K tile (M = 128 tokens), B = window rows (N = n_h per half).
 template <int D, int PASS>
 __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* sm, const Bars& b, int stages,
-                      int q_rows, const JobTable& jt)
+                      int q_rows, const JobTable& jt, uint32_t ones_stride)
 {
     const Shape& s = a.s;
     const int ntiles = (s.N + kTileTok - 1) / kTileTok;
@@ -295,7 +299,7 @@ __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* s
                 const uint32_t idesc = tc::idesc_bf16(128, jt.n(j));
                 const uint32_t qaddr = sbase + L.q + jt.row0(j) * 128;
                 if (PASS == 2)  // D = -lse2 / c per row (columns of D), then += K Q^T
-                    tc::umma_bf16(d_tmem, tc::sdesc_sw128(sbase + L.ones),
+                    tc::umma_bf16(d_tmem, tc::sdesc_sw128(sbase + L.ones, ones_stride),
                                   tc::sdesc_sw128(sbase + L.bias + 32 * j), idesc, 0);
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
@@ -336,7 +340,7 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
     const int group = (warp - 2) >> 2;   // which 32 tokens of each job
     const uint32_t tmem = tc::ld_shared(b.tmem_slot());
     float2* xchg = reinterpret_cast<float2*>(sm + L.xchg);  // [group - 1][rb][128]
-    const int nrb = q_rows / 128;
+    const int nrb = (q_rows + 127) / 128;
     const float c = kLog2e * rsqrtf((float)D);
     const unsigned long long c2 = tc::pack2(c, c);
     int c0, c1;
@@ -639,12 +643,13 @@ __global__ void lse_from_prefill_kernel(Shape s, LseTable t, float* __restrict__
 
 template <int D, int PASS>
 __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, int q_rows, int stages,
-                                                               int n_jobs, int granules)
+                                                               int n_jobs, int granules,
+                                                               int ones_atom)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-    const Smem L = smem_layout<D, PASS>(q_rows, stages);
+    const Smem L = smem_layout<D, PASS>(q_rows, stages, ones_atom != 0);
     const Bars b = bars_at(sm + L.bars, stages);
     const int warp = threadIdx.x >> 5;
     const JobTable jt = make_jobs(n_jobs, granules);
@@ -671,16 +676,19 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, int q_
         tc::tmem_relinquish();
     }
     if (PASS == 2 && threadIdx.x >= 64 && threadIdx.x < 64 + 128) {
-        // constant operand: 1 in columns 0-2 of every token row; the bias
-        // operand starts zeroed (the producer fills columns 16 j .. 16 j + 2)
+        // constant operand: 1 in columns 0-2 of every token row (one atom of
+        // 8 rows when ones_atom); the bias operand starts zeroed (the
+        // producer fills columns 16 j .. 16 j + 2)
         const int row = threadIdx.x - 64;
-        uint4* ones = reinterpret_cast<uint4*>(sm + L.ones + row * 128);
         uint4* bias = reinterpret_cast<uint4*>(sm + L.bias + row * 128);
-        for (int q = 0; q < 8; ++q) ones[q] = bias[q] = make_uint4(0u, 0u, 0u, 0u);
-        const uint32_t off = sw128_offset(row, 0) - (uint32_t)row * 128u;
-        uint8_t* r = sm + L.ones + row * 128 + off;
-        *reinterpret_cast<uint32_t*>(r) = 0x3F803F80u;  // bf16 1.0, 1.0
-        *reinterpret_cast<uint32_t*>(r + 4) = 0x00003F80u;
+        for (int q = 0; q < 8; ++q) bias[q] = make_uint4(0u, 0u, 0u, 0u);
+        if (!ones_atom || row < 8) {
+            uint4* ones = reinterpret_cast<uint4*>(sm + L.ones + row * 128);
+            for (int q = 0; q < 8; ++q) ones[q] = make_uint4(0u, 0u, 0u, 0u);
+            uint8_t* r = sm + L.ones + sw128_offset(row, 0);
+            *reinterpret_cast<uint32_t*>(r) = 0x3F803F80u;  // bf16 1.0, 1.0
+            *reinterpret_cast<uint32_t*>(r + 4) = 0x00003F80u;
+        }
         tc::fence_proxy_async_smem();
     }
     tc::fence_before_sync();
@@ -690,7 +698,7 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, int q_
     if (warp == 0) {
         produce<D, PASS>(a, L, sm, b, stages, q_rows, jt);
     } else if (warp == 1) {
-        if (tc::elect_one()) issue<D, PASS>(a, L, sm, b, stages, q_rows, jt);
+        if (tc::elect_one()) issue<D, PASS>(a, L, sm, b, stages, q_rows, jt, ones_atom ? 0u : 1024u);
     } else {
         if (PASS == 1)
             epilogue_stats<D>(a, L, sm, b, q_rows);
@@ -728,13 +736,18 @@ cudaError_t launch_impl(const TcArgs& a, cudaStream_t st)
 {
     const int rows = a.s.rows;
     // pass 1: whole 128-row MMA blocks; pass 2: whole 64-row TMA boxes
-    const int q_rows = PASS == 1 ? (rows + 127) / 128 * 128 : (rows + kQBox - 1) / kQBox * kQBox;
-    const int granules = PASS == 1 ? q_rows / 16 : (rows + 15) / 16;
-    const int n_jobs = PASS == 1 ? q_rows / 128 : (granules + 7) / 8;
+    // window rows in shared memory: whole 64-row TMA boxes.  Pass 1 runs
+    // whole 128-row MMA blocks over them; the last block's rows beyond
+    // q_rows read the next shared-memory region and their statistics are
+    // dropped (they are not window rows).
+    const int q_rows = (rows + kQBox - 1) / kQBox * kQBox;
+    const int n_jobs = PASS == 1 ? (q_rows + 127) / 128 : ((rows + 15) / 16 + 7) / 8;
+    const int granules = PASS == 1 ? 8 * n_jobs : (rows + 15) / 16;
     int stages = 4;
     const size_t budget = 227 * 1024 - 1024;
     while (stages > 2 && smem_layout<D, PASS>(q_rows, stages).total > budget) --stages;
-    const Smem L = smem_layout<D, PASS>(q_rows, stages);
+    const int ones_atom = smem_layout<D, PASS>(q_rows, stages).total > budget ? 1 : 0;
+    const Smem L = smem_layout<D, PASS>(q_rows, stages, ones_atom != 0);
     if (L.total > budget) return cudaErrorInvalidValue;
     // at least half of the SM's shared memory: one CTA (and one 512-column
     // TMEM allocation) per SM
@@ -744,7 +757,8 @@ cudaError_t launch_impl(const TcArgs& a, cudaStream_t st)
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
     if (e != cudaSuccess) return e;
     const int grid = a.total_chunks < num_sms() ? a.total_chunks : num_sms();
-    window_tc_kernel<D, PASS><<<grid, kThreads, bytes, st>>>(a, q_rows, stages, n_jobs, granules);
+    window_tc_kernel<D, PASS><<<grid, kThreads, bytes, st>>>(a, q_rows, stages, n_jobs, granules,
+                                                             ones_atom);
     return cudaGetLastError();
 }
 
