@@ -49,29 +49,38 @@ struct Smem {
     uint32_t total;
 };
 
+// How a launch cuts the work: the window rows in shared memory (whole 64-row
+// TMA boxes), the jobs of a tile (n_jobs jobs over `granules` 16-row
+// granules), the number of K stages and of TMEM accumulator buffers
+// (2^nbuf_log2 buffers of 512 >> nbuf_log2 columns).
+//
 // Pass 2 adds two bf16 operands in the same swizzled layout: a constant one
 // for every token (columns 0-2) and, per job j, the row bias -lse2 / c split
 // into three bf16 parts (columns 16 j .. 16 j + 2), so that one extra
 // K = 16 MMA subtracts each row's normaliser inside the accumulator.  The
-// bias operand has 128 rows x 64 columns.  The constant operand is 128
-// identical rows; when shared memory is short (512 window rows of d = 128)
-// only its first 8-row atom is stored and the descriptor's 8-row stride is
-// zero, so every group of 8 token rows reads the same atom.
-constexpr uint32_t kBiasOperandBytes = 128u * 128u;
+// bias operand has bias_rows rows (the largest job) x 64 columns.  The
+// constant operand is 128 identical rows; when shared memory is short only
+// its first 8-row atom is stored and its descriptor's 8-row stride is zero,
+// so every group of 8 token rows reads the same atom.
+struct Plan {
+    int q_rows, n_jobs, granules, stages, nbuf_log2, bias_rows, ones_atom;
+};
+
+constexpr uint32_t kOnesBytes = 128u * 128u;
 constexpr uint32_t kOnesAtomBytes = 8u * 128u;
 
 template <int D, int PASS>
-__host__ __device__ inline Smem smem_layout(int q_rows, int stages, bool ones_atom = false)
+__host__ __device__ inline Smem smem_layout(const Plan& p)
 {
     Smem s;
     constexpr int H = D / 64;
-    s.q_half = (uint32_t)q_rows * 128u;
+    s.q_half = (uint32_t)p.q_rows * 128u;
     s.k_stage = (uint32_t)H * kTileTok * 128u;
     s.q = 0;
     s.k = s.q + H * s.q_half;
-    s.ones = s.k + (uint32_t)stages * s.k_stage;
-    s.bias = s.ones + (PASS == 2 ? (ones_atom ? kOnesAtomBytes : kBiasOperandBytes) : 0u);
-    s.xchg = s.bias + (PASS == 2 ? kBiasOperandBytes : 0u);
+    s.ones = s.k + (uint32_t)p.stages * s.k_stage;
+    s.bias = s.ones + (PASS == 2 ? (p.ones_atom ? kOnesAtomBytes : kOnesBytes) : 0u);
+    s.xchg = s.bias + (PASS == 2 ? (uint32_t)p.bias_rows * 128u : 0u);
     // partials of groups 1.. (pass 1: per row block; pass 2: two tiles) + flags
     s.bars = s.xchg + (kGroups - 1) * (PASS == 1 ? 4u : 2u) * 128u * 8u + 64u;
     s.bars = (s.bars + 7u) & ~7u;
@@ -259,16 +268,16 @@ __device__ __forceinline__ void produce(const TcArgs& a, const Smem& L, uint8_t*
 
 // Pass 1: A = window rows (M = 128 per row block), B = K tile (N = 128).
 // Pass 2: A = K tile (M = 128 tokens), B = window rows (N = n_h per half).
-template <int D, int PASS>
+template <int D, int PASS, int NBUF_LOG2>
 __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* sm, const Bars& b, int stages,
-                      int q_rows, const JobTable& jt, uint32_t ones_stride)
+                      const JobTable& jt, uint32_t ones_stride)
 {
     const Shape& s = a.s;
     const int ntiles = (s.N + kTileTok - 1) / kTileTok;
     const uint32_t tmem = tc::ld_shared(b.tmem_slot());
     const uint32_t sbase = smem_u32(sm);
-    constexpr int NBUF = 4;
-    constexpr int BUF_COLS = 128;
+    constexpr int buf_mask = (1 << NBUF_LOG2) - 1;
+    constexpr uint32_t buf_cols = (uint32_t)kTmemCols >> NBUF_LOG2;
     int c0, c1;
     chunk_range(a.total_chunks, &c0, &c1);
     int cur_u = -1, qwaits = 0, kt = 0, job = 0;
@@ -291,11 +300,11 @@ __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* s
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 if (j >= jt.n_jobs) break;
-                const int buf = job % NBUF, nb = job / NBUF;
+                const int buf = job & buf_mask, nb = job >> NBUF_LOG2;
                 ++job;
                 if (!tc::mbar_wait(b.t_empty(buf), (nb & 1) ^ 1, b.abort())) { ok = false; break; }
                 tc::fence_after_sync();
-                const uint32_t d_tmem = tmem + buf * BUF_COLS;
+                const uint32_t d_tmem = tmem + buf * buf_cols;
                 const uint32_t idesc = tc::idesc_bf16(128, jt.n(j));
                 const uint32_t qaddr = sbase + L.q + jt.row0(j) * 128;
                 if (PASS == 2)  // D = -lse2 / c per row (columns of D), then += K Q^T
@@ -321,7 +330,6 @@ __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* s
     // every MMA issued must complete before TMEM is released
     tc::umma_commit(b.drain());
     tc::mbar_wait(b.drain(), 0, 0u);
-    (void)q_rows;
 }
 
 // ------------------------------------------------- epilogue, pass 1 (stats)
@@ -491,27 +499,37 @@ __device__ __forceinline__ void score_slice(float* v, int r0, int tok, const Sco
     }
 }
 
-template <bool FASTQ, bool MASK>
+template <bool FASTQ, bool MASK, int NBUF_LOG2>
 __device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int group, uint32_t tl,
                                            const Bars& b, const ScoreCtx& k, int tok,
                                            unsigned long long* bacc, float& qacc)
 {
     const int lane = threadIdx.x & 31;
+    constexpr uint32_t buf_cols = (uint32_t)kTmemCols >> NBUF_LOG2;
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
         if (j >= jt.n_jobs) break;
-        const int buf = job & 3, nb = job >> 2;
+        const int buf = job & ((1 << NBUF_LOG2) - 1), nb = job >> NBUF_LOG2;
         const int sl = (group + job) & (kGroups - 1);
         ++job;
         if (!tc::mbar_wait(b.t_full(buf), nb & 1, b.abort())) return false;
         tc::fence_after_sync();
         const int np = jt.n(j) >> 4, ns = (np + 1) >> 1;
-        const uint32_t taddr = tl + buf * 128 + 32 * sl;
-        const int r0 = jt.row0(j) + 32 * sl;
-        const bool mine = sl < ns, two = 2 * sl + 1 < np;
-        if (!MASK) {
-            float v[32];
-            if (mine) {
+        // this group's 32-column slices of the job: sl, sl + 4, ...; the
+        // buffer is released once the last of them is in registers
+        const int mine = sl < ns ? (sl + kGroups < ns ? 2 : 1) : 0;
+        if (mine == 0) {
+            tc::fence_before_sync();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
+        }
+        for (int q = 0; q < mine; ++q) {
+            const int sx = sl + kGroups * q;
+            const uint32_t taddr = tl + buf * buf_cols + 32 * sx;
+            const int r0 = jt.row0(j) + 32 * sx;
+            const bool two = 2 * sx + 1 < np, last = q + 1 == mine;
+            if (!MASK) {
+                float v[32];
                 if (two) {
                     tc::tmem_ld32(taddr, v);
                     tc::tmem_ld_wait_regs32(v);
@@ -519,34 +537,36 @@ __device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int gro
                     tc::tmem_ld16(taddr, v);
                     tc::tmem_ld_wait_regs16(v);
                 }
-            }
-            tc::fence_before_sync();
-            __syncwarp();
-            if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
-            if (mine) {
+                if (last) {
+                    tc::fence_before_sync();
+                    __syncwarp();
+                    if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
+                }
                 if (two)
                     score_slice<32, FASTQ, false>(v, r0, tok, k, bacc, qacc);
                 else
                     score_slice<16, FASTQ, false>(v, r0, tok, k, bacc, qacc);
+            } else {
+                // tiles that reach into the window (one or two per unit) go
+                // 16 columns at a time, keeping the masking's register demand low
+                float v[16];
+                for (int h = 0; h < (two ? 2 : 1); ++h) {
+                    tc::tmem_ld16(taddr + 16 * h, v);
+                    tc::tmem_ld_wait_regs16(v);
+                    score_slice<16, FASTQ, true>(v, r0 + 16 * h, tok, k, bacc, qacc);
+                }
+                if (last) {
+                    tc::fence_before_sync();
+                    __syncwarp();
+                    if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
+                }
             }
-        } else {
-            // tiles that reach into the window (one or two per unit) go 16
-            // columns at a time, keeping the masking's register demand low
-            float v[16];
-            for (int h = 0; h < (mine ? (two ? 2 : 1) : 0); ++h) {
-                tc::tmem_ld16(taddr + 16 * h, v);
-                tc::tmem_ld_wait_regs16(v);
-                score_slice<16, FASTQ, true>(v, r0 + 16 * h, tok, k, bacc, qacc);
-            }
-            tc::fence_before_sync();
-            __syncwarp();
-            if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
         }
     }
     return true;
 }
 
-template <int D, bool FASTQ>
+template <int D, bool FASTQ, int NBUF_LOG2>
 __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, uint8_t* sm,
                                                 const Bars& b, const JobTable& jt)
 {
@@ -577,8 +597,9 @@ __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, 
             const bool need_mask = t * kTileTok + kTileTok - 1 > s.N - s.W;
             unsigned long long bacc[2] = {0ull, 0ull};
             float qacc = 0.f;
-            ok = need_mask ? score_tile<FASTQ, true>(jt, job, group, tl, b, k, tok, bacc, qacc)
-                           : score_tile<FASTQ, false>(jt, job, group, tl, b, k, tok, bacc, qacc);
+            ok = need_mask
+                     ? score_tile<FASTQ, true, NBUF_LOG2>(jt, job, group, tl, b, k, tok, bacc, qacc)
+                     : score_tile<FASTQ, false, NBUF_LOG2>(jt, job, group, tl, b, k, tok, bacc, qacc);
             if (!ok) break;
             const float2 b2 = tc::unpack2(tc::add2(bacc[0], bacc[1]));
             float bsum = b2.x + b2.y;
@@ -642,20 +663,18 @@ __global__ void lse_from_prefill_kernel(Shape s, LseTable t, float* __restrict__
 // --------------------------------------------------------------- kernels
 
 template <int D, int PASS>
-__global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, int q_rows, int stages,
-                                                               int n_jobs, int granules,
-                                                               int ones_atom)
+__global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, Plan pl)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-    const Smem L = smem_layout<D, PASS>(q_rows, stages, ones_atom != 0);
-    const Bars b = bars_at(sm + L.bars, stages);
+    const Smem L = smem_layout<D, PASS>(pl);
+    const Bars b = bars_at(sm + L.bars, pl.stages);
     const int warp = threadIdx.x >> 5;
-    const JobTable jt = make_jobs(n_jobs, granules);
+    const JobTable jt = make_jobs(pl.n_jobs, pl.granules);
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < stages; ++i) {
+        for (int i = 0; i < pl.stages; ++i) {
             tc::mbar_init(b.k_full(i), 1);
             tc::mbar_init(b.k_empty(i), 1);
         }
@@ -680,9 +699,11 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, int q_
         // 8 rows when ones_atom); the bias operand starts zeroed (the
         // producer fills columns 16 j .. 16 j + 2)
         const int row = threadIdx.x - 64;
-        uint4* bias = reinterpret_cast<uint4*>(sm + L.bias + row * 128);
-        for (int q = 0; q < 8; ++q) bias[q] = make_uint4(0u, 0u, 0u, 0u);
-        if (!ones_atom || row < 8) {
+        for (int rr = row; rr < pl.bias_rows; rr += 128) {
+            uint4* bias = reinterpret_cast<uint4*>(sm + L.bias + rr * 128);
+            for (int q = 0; q < 8; ++q) bias[q] = make_uint4(0u, 0u, 0u, 0u);
+        }
+        if (!pl.ones_atom || row < 8) {
             uint4* ones = reinterpret_cast<uint4*>(sm + L.ones + row * 128);
             for (int q = 0; q < 8; ++q) ones[q] = make_uint4(0u, 0u, 0u, 0u);
             uint8_t* r = sm + L.ones + sw128_offset(row, 0);
@@ -696,16 +717,24 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, int q_
     tc::fence_after_sync();
 
     if (warp == 0) {
-        produce<D, PASS>(a, L, sm, b, stages, q_rows, jt);
+        produce<D, PASS>(a, L, sm, b, pl.stages, pl.q_rows, jt);
     } else if (warp == 1) {
-        if (tc::elect_one()) issue<D, PASS>(a, L, sm, b, stages, q_rows, jt, ones_atom ? 0u : 1024u);
+        if (tc::elect_one()) {
+            const uint32_t ones_stride = pl.ones_atom ? 0u : 1024u;
+            if (pl.nbuf_log2 == 1)
+                issue<D, PASS, 1>(a, L, sm, b, pl.stages, jt, ones_stride);
+            else
+                issue<D, PASS, 2>(a, L, sm, b, pl.stages, jt, ones_stride);
+        }
     } else {
         if (PASS == 1)
-            epilogue_stats<D>(a, L, sm, b, q_rows);
+            epilogue_stats<D>(a, L, sm, b, pl.q_rows);
+        else if (a.s.W % 16 == 0 && pl.nbuf_log2 == 1)
+            epilogue_scores<D, true, 1>(a, L, sm, b, jt);
         else if (a.s.W % 16 == 0)
-            epilogue_scores<D, true>(a, L, sm, b, jt);
-        else
-            epilogue_scores<D, false>(a, L, sm, b, jt);
+            epilogue_scores<D, true, 2>(a, L, sm, b, jt);
+        else  // W % 16 != 0: always four accumulators (see launch_impl)
+            epilogue_scores<D, false, 2>(a, L, sm, b, jt);
     }
 
     tc::fence_before_sync();
@@ -735,20 +764,34 @@ template <int D, int PASS>
 cudaError_t launch_impl(const TcArgs& a, cudaStream_t st)
 {
     const int rows = a.s.rows;
-    // pass 1: whole 128-row MMA blocks; pass 2: whole 64-row TMA boxes
-    // window rows in shared memory: whole 64-row TMA boxes.  Pass 1 runs
-    // whole 128-row MMA blocks over them; the last block's rows beyond
-    // q_rows read the next shared-memory region and their statistics are
-    // dropped (they are not window rows).
-    const int q_rows = (rows + kQBox - 1) / kQBox * kQBox;
-    const int n_jobs = PASS == 1 ? (q_rows + 127) / 128 : ((rows + 15) / 16 + 7) / 8;
-    const int granules = PASS == 1 ? 8 * n_jobs : (rows + 15) / 16;
-    int stages = 4;
     const size_t budget = 227 * 1024 - 1024;
-    while (stages > 2 && smem_layout<D, PASS>(q_rows, stages).total > budget) --stages;
-    const int ones_atom = smem_layout<D, PASS>(q_rows, stages).total > budget ? 1 : 0;
-    const Smem L = smem_layout<D, PASS>(q_rows, stages, ones_atom != 0);
-    if (L.total > budget) return cudaErrorInvalidValue;
+    // window rows in shared memory: whole 64-row TMA boxes.  Pass 1 runs
+    // whole 128-row MMA blocks over them in four 128-column accumulators; the
+    // last block's rows beyond q_rows read the next shared-memory region and
+    // their statistics are dropped (they are not window rows).  Pass 2 cuts
+    // the rows into jobs of up to 256 rows (two 256-column accumulators, the
+    // more efficient MMA shape) when shared memory allows, else up to 128.
+    Plan pl;
+    pl.q_rows = (rows + kQBox - 1) / kQBox * kQBox;
+    const int granules = (rows + 15) / 16;
+    Smem L;
+    bool fits = false;
+    // (a window that is not a multiple of 16 rows always takes 128-row jobs)
+    for (int attempt = a.s.W % 16 == 0 ? 0 : 1; attempt < 2 && !fits; ++attempt) {
+        const int per_job = PASS == 1 ? 8 : (attempt == 0 ? 16 : 8);  // granules
+        pl.n_jobs = PASS == 1 ? (pl.q_rows + 127) / 128 : (granules + per_job - 1) / per_job;
+        pl.granules = PASS == 1 ? 8 * pl.n_jobs : granules;
+        pl.nbuf_log2 = per_job == 16 ? 1 : 2;
+        pl.bias_rows = PASS == 2 ? 16 * ((pl.granules + pl.n_jobs - 1) / pl.n_jobs) : 0;
+        for (pl.ones_atom = 0; pl.ones_atom < 2 && !fits; ++pl.ones_atom) {
+            for (pl.stages = 4; pl.stages > 2; --pl.stages)
+                if (smem_layout<D, PASS>(pl).total <= budget) break;
+            L = smem_layout<D, PASS>(pl);
+            fits = L.total <= budget;
+            if (fits) break;
+        }
+    }
+    if (!fits) return cudaErrorInvalidValue;
     // at least half of the SM's shared memory: one CTA (and one 512-column
     // TMEM allocation) per SM
     size_t bytes = L.total + 1024;
@@ -757,8 +800,7 @@ cudaError_t launch_impl(const TcArgs& a, cudaStream_t st)
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
     if (e != cudaSuccess) return e;
     const int grid = a.total_chunks < num_sms() ? a.total_chunks : num_sms();
-    window_tc_kernel<D, PASS><<<grid, kThreads, bytes, st>>>(a, q_rows, stages, n_jobs, granules,
-                                                             ones_atom);
+    window_tc_kernel<D, PASS><<<grid, kThreads, bytes, st>>>(a, pl);
     return cudaGetLastError();
 }
 
