@@ -3,13 +3,12 @@
 //
 // "The k best" always means: larger value first, equal values -> lower index
 // first.  Values are compared through order-preserving 32-bit keys
-// (float_key).  A radix select (4 x 8-bit digits, warp-aggregated histogram
-// updates) finds the k-th best key tau and how many elements equal to tau
-// are taken; index-ordered sweeps then decide membership: key > tau, or
-// key == tau among the first `need` equal keys.  The sweeps are
-// warp-segmented (warp w owns a contiguous index range, its lanes take
-// consecutive elements) so that reads are conflict-free while ballots keep
-// the index order inside a warp.
+// (float_key).  A range-adaptive radix select finds the k-th best key tau
+// and how many elements equal to tau are taken; index-ordered sweeps then
+// decide membership: key > tau, or key == tau among the first `need` equal
+// keys.  The sweeps are warp-segmented (warp w owns a contiguous index
+// range, its lanes take consecutive elements) so that reads are
+// conflict-free while ballots keep the index order inside a warp.
 //
 // A key accessor `key_of(i, key)` returns false for elements excluded from a
 // selection (they are neither counted nor taken).
@@ -25,62 +24,121 @@ struct SelectResult {
     int need;      // how many elements with key == tau are taken
 };
 
+// Histogram bins of one select pass (shared memory of the caller).
+constexpr int kSelBits = 11;
+constexpr int kSelBins = 1 << kSelBits;
+
 // k-th best key over the included elements of [0, n) (1 <= k <= their
-// count).  Every thread returns the same result.
+// count).  First the range [kmin, kmax] of the included keys, then passes
+// over it: each pass histograms the keys of the current range into
+// kSelBins bins of 2^shift keys (plain shared-memory adds: the bins follow
+// the data's own range, so few keys share one), takes the bin where the
+// count from the top reaches k, and narrows the range to it, until a bin is
+// one key.  At most three passes for 32-bit keys.  Every thread returns the
+// same result; blockDim.x must be 1024 (32 warps x 64 bins in the scan).
 template <typename KeyFn>
 __device__ SelectResult radix_select_by(int n, int k, KeyFn key_of, int* hist, int* bcast)
 {
-    uint32_t prefix = 0, mask = 0;
-    int remaining = k;
-    for (int shift = 24; shift >= 0; shift -= 8) {
-        for (int b = threadIdx.x; b < 256; b += blockDim.x) hist[b] = 0;
-        __syncthreads();
-        // warp-aggregated: lanes that fall into the same bin add once together
-        const int n_round = (n + 31) & ~31;
-        for (int i = threadIdx.x; i < n_round; i += blockDim.x) {
-            uint32_t key = 0u;
-            const bool in = i < n && key_of(i, key);
-            const bool hit = in && (key & mask) == prefix;
-            const int bin = hit ? (int)((key >> shift) & 255u) : -1;
-            const uint32_t peers = __match_any_sync(0xffffffffu, bin);
-            if (hit && (threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    uint32_t kmin = 0xffffffffu, kmax = 0u;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+        uint32_t key;
+        if (key_of(i, key)) {
+            kmin = min(kmin, key);
+            kmax = max(kmax, key);
         }
-        __syncthreads();
-        if (threadIdx.x < 32) {
-            // bins high to low: find the bin where the running count from the
-            // top reaches `remaining`
-            const int lane = threadIdx.x;
-            int cum = 0, found_bin = -1, found_rem = 0;
-            for (int base = 255; base >= 0 && found_bin < 0; base -= 32) {
-                const int b = base - lane;
-                const int c = hist[b];
-                int incl = c;  // inclusive scan from the top (lane 0 = highest bin)
-#pragma unroll
-                for (int o = 1; o < 32; o <<= 1) {
-                    const int y = __shfl_up_sync(0xffffffffu, incl, o);
-                    if (lane >= o) incl += y;
-                }
-                const uint32_t ballot = __ballot_sync(0xffffffffu, cum + incl >= remaining);
-                if (ballot) {
-                    const int first = __ffs(ballot) - 1;
-                    const int excl = __shfl_sync(0xffffffffu, incl - c, first);
-                    found_bin = base - first;
-                    found_rem = remaining - (cum + excl);
-                }
-                cum += __shfl_sync(0xffffffffu, incl, 31);
-            }
-            if (lane == 0) {
-                bcast[0] = found_bin;
-                bcast[1] = found_rem;
-            }
-        }
-        __syncthreads();
-        prefix |= (uint32_t)bcast[0] << shift;
-        mask |= 255u << shift;
-        remaining = bcast[1];
-        __syncthreads();
     }
-    return {prefix, remaining};
+    kmin = __reduce_min_sync(0xffffffffu, kmin);
+    kmax = __reduce_max_sync(0xffffffffu, kmax);
+    if (lane == 0) {
+        hist[warp] = (int)kmin;
+        hist[32 + warp] = (int)kmax;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        const uint32_t a = __reduce_min_sync(0xffffffffu, (uint32_t)hist[lane]);
+        const uint32_t b = __reduce_max_sync(0xffffffffu, (uint32_t)hist[32 + lane]);
+        if (lane == 0) {
+            bcast[0] = (int)a;
+            bcast[1] = (int)b;
+        }
+    }
+    __syncthreads();
+    uint32_t lo = (uint32_t)bcast[0];
+    const uint64_t span = (uint64_t)(uint32_t)bcast[1] - lo + 1u;
+    int shift = 0;
+    while (((span - 1u) >> shift) >= (uint64_t)kSelBins) ++shift;  // top bin index < kSelBins
+    uint64_t width = span;  // keys of the current range: [lo, lo + width)
+    int remaining = k;
+    __syncthreads();
+    while (true) {
+        for (int b = threadIdx.x; b < kSelBins; b += blockDim.x) hist[b] = 0;
+        __syncthreads();
+        for (int i0 = threadIdx.x; i0 < n; i0 += 4 * blockDim.x) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int i = i0 + q * (int)blockDim.x;
+                uint32_t key = 0u;
+                if (i < n && key_of(i, key) && key >= lo && (uint64_t)(key - lo) < width)
+                    atomicAdd(&hist[(key - lo) >> shift], 1);
+            }
+        }
+        __syncthreads();
+        // bins from the top: lane l of warp w holds bins 64 w + 63 - 2 l and
+        // 64 w + 62 - 2 l; warp totals first, then the boundary warp's bins
+        const int bhi = 64 * warp + 63 - 2 * lane;
+        const int chi = hist[bhi], clo = hist[bhi - 1];
+        int incl = chi + clo;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += y;
+        }
+        __syncthreads();  // everyone has read the bins
+        if (lane == 31) hist[kSelBins + warp] = incl;  // warp total
+        __syncthreads();
+        if (warp == 0) {
+            // warps from the top: above[w] = totals of warps w + 1 .. 31
+            const int tot = hist[kSelBins + 31 - lane];
+            int cum = tot;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(0xffffffffu, cum, o);
+                if (lane >= o) cum += y;
+            }
+            const uint32_t hit = __ballot_sync(0xffffffffu, cum >= remaining);
+            const int first = __ffs(hit) - 1;  // the boundary warp is 31 - first
+            const int above = __shfl_sync(0xffffffffu, cum - tot, first);
+            if (lane == 0) {
+                bcast[2] = 31 - first;
+                bcast[3] = above;
+            }
+        }
+        __syncthreads();
+        if (warp == bcast[2]) {
+            const int rem = remaining - bcast[3];
+            const uint32_t hit = __ballot_sync(0xffffffffu, incl >= rem);
+            const int first = __ffs(hit) - 1;
+            if (lane == first) {
+                const int before = incl - chi - clo;  // bins above this lane's pair
+                if (before + chi >= rem) {
+                    bcast[0] = bhi;
+                    bcast[1] = rem - before;
+                } else {
+                    bcast[0] = bhi - 1;
+                    bcast[1] = rem - before - chi;
+                }
+            }
+        }
+        __syncthreads();
+        lo += (uint32_t)bcast[0] << shift;
+        remaining = bcast[1];
+        width = (uint64_t)1 << shift;
+        __syncthreads();
+        if (shift == 0) break;
+        shift = shift > kSelBits ? shift - kSelBits : 0;
+    }
+    return {lo, remaining};
 }
 
 struct Segment {
