@@ -24,7 +24,7 @@ adaptive_select_kernel(Shape s, int keep_window, AdaptArgs a)
 {
     extern __shared__ uint8_t taken[];  // [Hkv][n_cand]
     __shared__ int hist[kSelBins + 32];
-    __shared__ int bcast[4];
+    __shared__ int bcast[8];
     __shared__ int warp_sums[32];
     __shared__ int total_s;
 
@@ -49,7 +49,7 @@ adaptive_select_kernel(Shape s, int keep_window, AdaptArgs a)
                 const float* Sh = Sp + (size_t)h * N;
                 const SelectResult r = radix_select(Sh, n_cand, g, hist, bcast);
                 const Segment sg = warp_segment(n_cand);
-                const int eqb = eq_before_segment(Sh, sg, r.tau, warp_sums, &total_s);
+                const int eqb = eq_before_segment(Sh, sg, r, warp_sums, &total_s);
                 walk_topk(Sh, sg, r, eqb, [&](int i, bool, bool in) {
                     if (in) taken[h * n_cand + i] = 1;
                 });
@@ -67,7 +67,7 @@ adaptive_select_kernel(Shape s, int keep_window, AdaptArgs a)
             };
             const SelectResult r = radix_select_by(total, rest, key_of, hist, bcast);
             const Segment sg = warp_segment(total);
-            const int eqb = eq_before_segment_by(sg, r.tau, key_of, warp_sums, &total_s);
+            const int eqb = eq_before_segment_by(sg, r, key_of, warp_sums, &total_s);
             // a warp only marks its own segment, after evaluating each element
             walk_topk_by(sg, r, eqb, key_of, [&](int f, bool, bool in) {
                 if (in) taken[f] = 1;

@@ -40,6 +40,37 @@ __device__ float block_sum(float v, float* red)
     return tot;
 }
 
+// Four block-wide fp32 sums in one round (red holds 4 x 33 floats).
+__device__ float4 block_sum4(float4 v, float* red)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        v.x += __shfl_xor_sync(0xffffffffu, v.x, o);
+        v.y += __shfl_xor_sync(0xffffffffu, v.y, o);
+        v.z += __shfl_xor_sync(0xffffffffu, v.z, o);
+        v.w += __shfl_xor_sync(0xffffffffu, v.w, o);
+    }
+    if (lane == 0) {
+        red[warp] = v.x;
+        red[33 + warp] = v.y;
+        red[66 + warp] = v.z;
+        red[99 + warp] = v.w;
+    }
+    __syncthreads();
+    if (warp < 4) {
+        const int nw = (int)(blockDim.x >> 5);
+        float t = lane < nw ? red[33 * warp + lane] : 0.f;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        if (lane == 0) red[33 * warp + 32] = t;
+    }
+    __syncthreads();
+    const float4 tot = make_float4(red[32], red[65], red[98], red[131]);
+    __syncthreads();
+    return tot;
+}
+
 // dst[0, n) = src[0, n) with independent 16-byte loads (n % 4 == 0 and both
 // 16-byte aligned), so the copy costs a few memory round trips, not one per
 // element.
@@ -69,9 +100,9 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
     float* Sb = sm;      // pooled backbone B~, then the final score S
     float* Vs = sm + N;  // calibrated evidence V
     __shared__ int hist[kSelBins + 32];
-    __shared__ int bcast[4];
+    __shared__ int bcast[8];
     __shared__ int warp_sums[32];
-    __shared__ float red[33];
+    __shared__ float red[4 * 33];
     __shared__ int total_s;
 
     const int pair = u / s.hkv, h = u - pair * s.hkv;
@@ -82,6 +113,7 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
     const int kept_total = min(a.budget[pair], N);
     const int keep = kept_total - win;
 
+    uint32_t skmin = 0xffffffffu, skmax = 0u;  // key range of S over the candidates
     auto Eof = [&](int j) -> const float* {
         return a.Ering + (long long)rq * a.ring_req_stride +
                (long long)(j % a.ring) * s.hkv * N + (long long)h * N;
@@ -99,12 +131,15 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
         else
             for (int i = threadIdx.x; i < N; i += blockDim.x) Vs[i] = Bu[i];
         __syncthreads();
+        uint32_t kmin = 0xffffffffu, kmax = 0u;  // key range of B~ over the candidates
         for (int i = threadIdx.x; i < N; i += blockDim.x) {
             float mx = 0.f;
             if (i < n_cand) {
                 mx = -INFINITY;
                 const int lo = max(0, i - half), hi = min(n_cand - 1, i + half);
                 for (int v = lo; v <= hi; ++v) mx = fmaxf(mx, Vs[v]);
+                kmin = min(kmin, float_key(mx));
+                kmax = max(kmax, float_key(mx));
             }
             Sb[i] = mx;
         }
@@ -147,10 +182,12 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
             }
         }
         __syncthreads();
+        float vsum = 0.f;  // over the candidates: the shift of the moments below
 #pragma unroll
         for (int k = 0; k < kMaxPer; ++k) {
             const int i = threadIdx.x + k * blockDim.x;
             if (i < N) Vs[i] = vreg[k];
+            if (i < n_cand) vsum += vreg[k];
         }
         __syncthreads();
         if (a.V) for (int i = threadIdx.x; i < N; i += blockDim.x) a.V[(size_t)u * N + i] = Vs[i];
@@ -162,32 +199,43 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
         const int M = (int)(Ml < n_cand ? Ml : n_cand);
         float lam = 0.f;
         if (M > 0) {
-            const SelectResult sel = radix_select(Sb, n_cand, M, hist, bcast);
+            const SelectResult sel =
+                radix_select_range(n_cand, M, FloatKeys{Sb}, hist, bcast, kmin, kmax);
             const Segment sg = warp_segment(n_cand);
-            const int eqb = eq_before_segment(Sb, sg, sel.tau, warp_sums, &total_s);
-            float sb = 0.f, sv = 0.f;
+            const int eqb = eq_before_segment(Sb, sg, sel, warp_sums, &total_s);
+            // moments about fixed shifts in one walk: B~ about its M-th value,
+            // V about its mean over the candidates (both near the members'
+            // means, so the fp32 differences keep their precision)
+            const float pb = key_float(sel.tau);
+            const float pv = block_sum(vsum, red) / (float)n_cand;
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
             walk_topk(Sb, sg, sel, eqb, [&](int i, bool, bool in) {
                 if (in) {
-                    sb += Sb[i];
-                    sv += Vs[i];
+                    const float db = Sb[i] - pb, dv = Vs[i] - pv;
+                    acc.x += db;
+                    acc.y = fmaf(db, db, acc.y);
+                    acc.z += dv;
+                    acc.w = fmaf(dv, dv, acc.w);
                 }
             });
-            const float mb = block_sum(sb, red) / (float)M;
-            const float mv = block_sum(sv, red) / (float)M;
-            float vb = 0.f, vv = 0.f;  // centred second moments (two-pass)
-            walk_topk(Sb, sg, sel, eqb, [&](int i, bool, bool in) {
-                if (in) {
-                    const float db = Sb[i] - mb, dv = Vs[i] - mv;
-                    vb = fmaf(db, db, vb);
-                    vv = fmaf(dv, dv, vv);
-                }
-            });
-            const float stdb = sqrtf(block_sum(vb, red) / (float)M);
-            const float stdv = sqrtf(block_sum(vv, red) / (float)M);
+            const float4 tot = block_sum4(acc, red);
+            const float inv_m = 1.f / (float)M;
+            const float mb = tot.x * inv_m, mv = tot.z * inv_m;
+            const float stdb = sqrtf(fmaxf(tot.y * inv_m - mb * mb, 0.f));
+            const float stdv = sqrtf(fmaxf(tot.w * inv_m - mv * mv, 0.f));
             lam = c.gamma * stdb / (stdv + c.eps);
         }
         if (threadIdx.x == 0 && lam_out) *lam_out = lam;
-        for (int i = threadIdx.x; i < n_cand; i += blockDim.x) Sb[i] = fmaf(lam, Vs[i], Sb[i]);
+        kmin = 0xffffffffu;
+        kmax = 0u;
+        for (int i = threadIdx.x; i < n_cand; i += blockDim.x) {
+            const float sv = fmaf(lam, Vs[i], Sb[i]);
+            Sb[i] = sv;
+            kmin = min(kmin, float_key(sv));
+            kmax = max(kmax, float_key(sv));
+        }
+        skmin = kmin;
+        skmax = kmax;
         __syncthreads();
         if (a.write_S)
             for (int i = threadIdx.x; i < N; i += blockDim.x) a.S[(size_t)u * N + i] = Sb[i];
@@ -197,13 +245,19 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
     }
 
     if (!a.do_select) return;
+    if (!a.compute_scores)
+        for (int i = threadIdx.x; i < n_cand; i += blockDim.x) {
+            skmin = min(skmin, float_key(Sb[i]));
+            skmax = max(skmax, float_key(Sb[i]));
+        }
     int32_t* out = idx_pair + (size_t)h * kept_total;
     if (keep >= n_cand) {
         for (int i = threadIdx.x; i < n_cand; i += blockDim.x) out[i] = i;
     } else if (keep > 0) {
-        const SelectResult sel = radix_select(Sb, n_cand, keep, hist, bcast);
+        const SelectResult sel =
+            radix_select_range(n_cand, keep, FloatKeys{Sb}, hist, bcast, skmin, skmax);
         const Segment sg = warp_segment(n_cand);
-        const int eqb = eq_before_segment(Sb, sg, sel.tau, warp_sums, &total_s);
+        const int eqb = eq_before_segment(Sb, sg, sel, warp_sums, &total_s);
         int mine = 0;
         walk_topk(Sb, sg, sel, eqb, [&](int, bool, bool in) { mine += in; });
         const int base = warp_exclusive_scan(warp_sum(mine), warp_sums, &total_s);

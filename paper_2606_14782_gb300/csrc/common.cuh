@@ -53,11 +53,15 @@ __device__ __forceinline__ float fast_exp2(float x)
 }
 
 // Order-preserving map of a float to an unsigned key (larger float ->
-// larger key), used by the radix selections.
+// larger key), used by the radix selections, and its inverse.
 __device__ __forceinline__ uint32_t float_key(float f)
 {
     uint32_t b = __float_as_uint(f);
     return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+__device__ __forceinline__ float key_float(uint32_t k)
+{
+    return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
 }
 
 // ----------------------------------------------------------- launchers

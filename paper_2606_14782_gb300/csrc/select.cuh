@@ -22,6 +22,10 @@ namespace sel {
 struct SelectResult {
     uint32_t tau;  // key of the k-th best element
     int need;      // how many elements with key == tau are taken
+    int count_eq;  // how many included elements have key == tau
+    // every element equal to tau is taken: membership is key >= tau and
+    // needs no index-ordered counting
+    __device__ __forceinline__ bool all_ties_in() const { return need == count_eq; }
 };
 
 // Histogram bins of one select pass (shared memory of the caller).
@@ -36,18 +40,13 @@ constexpr int kSelBins = 1 << kSelBits;
 // count from the top reaches k, and narrows the range to it, until a bin is
 // one key.  At most three passes for 32-bit keys.  Every thread returns the
 // same result; blockDim.x must be 1024 (32 warps x 64 bins in the scan).
+// kmin / kmax: this thread's share of the key range (the callers that know
+// it from an earlier pass over the keys pass it in; see radix_select_by).
 template <typename KeyFn>
-__device__ SelectResult radix_select_by(int n, int k, KeyFn key_of, int* hist, int* bcast)
+__device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist, int* bcast,
+                                           uint32_t kmin, uint32_t kmax)
 {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    uint32_t kmin = 0xffffffffu, kmax = 0u;
-    for (int i = threadIdx.x; i < n; i += blockDim.x) {
-        uint32_t key;
-        if (key_of(i, key)) {
-            kmin = min(kmin, key);
-            kmax = max(kmax, key);
-        }
-    }
     kmin = __reduce_min_sync(0xffffffffu, kmin);
     kmax = __reduce_max_sync(0xffffffffu, kmax);
     if (lane == 0) {
@@ -124,21 +123,37 @@ __device__ SelectResult radix_select_by(int n, int k, KeyFn key_of, int* hist, i
                 if (before + chi >= rem) {
                     bcast[0] = bhi;
                     bcast[1] = rem - before;
+                    bcast[4] = chi;
                 } else {
                     bcast[0] = bhi - 1;
                     bcast[1] = rem - before - chi;
+                    bcast[4] = clo;
                 }
             }
         }
         __syncthreads();
         lo += (uint32_t)bcast[0] << shift;
         remaining = bcast[1];
+        const int in_bin = bcast[4];
         width = (uint64_t)1 << shift;
         __syncthreads();
-        if (shift == 0) break;
+        if (shift == 0) return {lo, remaining, in_bin};
         shift = shift > kSelBits ? shift - kSelBits : 0;
     }
-    return {lo, remaining};
+}
+
+template <typename KeyFn>
+__device__ SelectResult radix_select_by(int n, int k, KeyFn key_of, int* hist, int* bcast)
+{
+    uint32_t kmin = 0xffffffffu, kmax = 0u;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+        uint32_t key;
+        if (key_of(i, key)) {
+            kmin = min(kmin, key);
+            kmax = max(kmax, key);
+        }
+    }
+    return radix_select_range(n, k, key_of, hist, bcast, kmin, kmax);
 }
 
 struct Segment {
@@ -186,11 +201,14 @@ __device__ inline int warp_exclusive_scan(int v, int* warp_sums, int* total)
     return r;
 }
 
-// Included keys equal to tau before this warp's segment.
+// Included keys equal to tau before this warp's segment (0 without a pass
+// when every tie is taken: the walks then never need the count).
 template <typename KeyFn>
-__device__ int eq_before_segment_by(Segment sg, uint32_t tau, KeyFn key_of, int* warp_sums,
+__device__ int eq_before_segment_by(Segment sg, SelectResult sel, KeyFn key_of, int* warp_sums,
                                     int* total)
 {
+    if (sel.all_ties_in()) return 0;
+    const uint32_t tau = sel.tau;
     int eq = 0;
     for (int i = sg.lo + (threadIdx.x & 31); i < sg.hi; i += 32) {
         uint32_t key = 0u;
@@ -236,10 +254,10 @@ __device__ inline SelectResult radix_select(const float* vals, int n, int k, int
 {
     return radix_select_by(n, k, FloatKeys{vals}, hist, bcast);
 }
-__device__ inline int eq_before_segment(const float* vals, Segment sg, uint32_t tau,
+__device__ inline int eq_before_segment(const float* vals, Segment sg, SelectResult sel,
                                         int* warp_sums, int* total)
 {
-    return eq_before_segment_by(sg, tau, FloatKeys{vals}, warp_sums, total);
+    return eq_before_segment_by(sg, sel, FloatKeys{vals}, warp_sums, total);
 }
 template <typename F>
 __device__ __forceinline__ void walk_topk(const float* vals, Segment sg, SelectResult sel,
