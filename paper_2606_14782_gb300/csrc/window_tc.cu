@@ -81,15 +81,16 @@ __host__ __device__ inline Smem smem_layout(const Plan& p)
     s.ones = s.k + (uint32_t)p.stages * s.k_stage;
     s.bias = s.ones + (PASS == 2 ? (p.ones_atom ? kOnesAtomBytes : kOnesBytes) : 0u);
     s.xchg = s.bias + (PASS == 2 ? (uint32_t)p.bias_rows * 128u : 0u);
-    // partials of groups 1.. (pass 1: per row block; pass 2: two tiles) + flags
-    s.bars = s.xchg + (kGroups - 1) * (PASS == 1 ? 4u : 2u) * 128u * 8u + 64u;
+    // pass 1: partials of groups 1.. per row block; pass 2: every group's
+    // partial sums for four tiles; then per-tile arrival counters / flags
+    s.bars = s.xchg + (PASS == 1 ? (kGroups - 1) * 4u * 128u * 8u : 4u * kGroups * 128u * 8u) + 64u;
     s.bars = (s.bars + 7u) & ~7u;
     s.total = s.bars + 256u;  // barriers, TMEM base, abort flag
     return s;
 }
 
 // Barrier block, 8-byte slots from `base` (a shared-memory address):
-// t_full[4], t_empty[4], q_full, q_empty, drain, ep_all, ep_pair[4], the
+// t_full[4], t_empty[4], q_full, q_empty, drain, ep_all, four spare slots, the
 // TMEM base word, the abort word, then k_full[stages], k_empty[stages].
 struct Bars {
     uint32_t base;
@@ -100,8 +101,6 @@ struct Bars {
     __device__ __forceinline__ uint32_t q_empty() const { return base + 72u; }
     __device__ __forceinline__ uint32_t drain() const { return base + 80u; }
     __device__ __forceinline__ uint32_t ep_all() const { return base + 88u; }
-    // the epilogue warps of one TMEM lane quarter
-    __device__ __forceinline__ uint32_t ep_pair(int q) const { return base + 96u + 8u * q; }
     __device__ __forceinline__ uint32_t tmem_slot() const { return base + 128u; }
     __device__ __forceinline__ uint32_t abort() const { return base + 136u; }
     __device__ __forceinline__ uint32_t k_full(int st) const { return base + 144u + 8u * st; }
@@ -576,7 +575,8 @@ __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, 
     const int quarter = warp & 3;
     const int group = (warp - 2) >> 2;
     const uint32_t tl = tc::ld_shared(b.tmem_slot()) + ((uint32_t)(quarter * 32) << 16);
-    float2* xs = reinterpret_cast<float2*>(sm + L.xchg);  // [2][kGroups - 1][128]
+    float2* xs = reinterpret_cast<float2*>(sm + L.xchg);  // [4][kGroups][128]
+    int* cnt = reinterpret_cast<int*>(xs + 4 * kGroups * 128);  // [4 tiles][4 quarters]
     ScoreCtx k;
     const float c = kLog2e * rsqrtf((float)D);
     k.c2 = tc::pack2(c, c);
@@ -587,7 +587,7 @@ __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, 
         if (16 * g + 15 < s.rows && (16 * g + 15) % s.W == s.W - 1) k.qmask |= 1u << g;
     int c0, c1;
     chunk_range(a.total_chunks, &c0, &c1);
-    int job = 0, pair_phase = 0;
+    int job = 0;
     bool ok = true;
     for (int g = c0; g < c1 && ok; ++g) {
         const int u = g / a.chunks, ci = g - u * a.chunks;
@@ -604,21 +604,36 @@ __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, 
             const float2 b2 = tc::unpack2(tc::add2(bacc[0], bacc[1]));
             float bsum = b2.x + b2.y;
             float qsum = qacc * (float)s.W;
-            // the groups' partial sums of a token meet in shared memory
-            // (double-buffered by tile)
-            float2* slots = xs + (t & 1) * (kGroups - 1) * 128 + quarter * 32 + lane;
-            if (group > 0) slots[(group - 1) * 128] = make_float2(bsum, qsum);
-            if (!warp_barrier(b.ep_pair(quarter), pair_phase, b.abort())) { ok = false; break; }
-            if (group == 0 && tok < s.N) {
-                for (int gg = 0; gg < kGroups - 1; ++gg) {
-                    const float2 o = slots[gg * 128];
-                    bsum += o.x;
-                    qsum += o.y;
+            // the groups' partial sums of a token meet in shared memory,
+            // four tile slots deep; the last group to arrive adds them in
+            // group order and stores the token's B, Q and E
+            float2* slot = xs + (size_t)((t & 3) * kGroups) * 128 + quarter * 32 + lane;
+            slot[group * 128] = make_float2(bsum, qsum);
+            __syncwarp();
+            int last = 0;
+            if (lane == 0) {
+                __threadfence_block();
+                last = atomicAdd(cnt + (t & 3) * 4 + quarter, 1) == kGroups - 1;
+            }
+            last = __shfl_sync(0xffffffffu, last, 0);
+            if (last) {
+                __threadfence_block();
+                const volatile float2* vs = slot;
+                float2 o = make_float2(vs[0].x, vs[0].y);
+                bsum = o.x;
+                qsum = o.y;
+                for (int gg = 1; gg < kGroups; ++gg) {
+                    bsum += vs[gg * 128].x;
+                    qsum += vs[gg * 128].y;
                 }
-                const size_t idx = (size_t)u * s.N + tok;
-                a.B[idx] = bsum;
-                a.Q[idx] = qsum;
-                a.E[idx] = fmaxf(qsum - bsum, 0.f);
+                if (tok < s.N) {
+                    const size_t idx = (size_t)u * s.N + tok;
+                    a.B[idx] = bsum;
+                    a.Q[idx] = qsum;
+                    a.E[idx] = fmaxf(qsum - bsum, 0.f);
+                }
+                __syncwarp();
+                if (lane == 0) cnt[(t & 3) * 4 + quarter] = 0;
             }
         }
     }
@@ -686,7 +701,6 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, Plan p
         tc::mbar_init(b.q_empty(), 1);
         tc::mbar_init(b.drain(), 1);
         tc::mbar_init(b.ep_all(), kEpiThreads / 32);
-        for (int i = 0; i < 4; ++i) tc::mbar_init(b.ep_pair(i), kGroups);
         tc::st_shared_volatile(b.abort(), 0u);
         tc::fence_barrier_init();
     }
@@ -703,6 +717,7 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, Plan p
             uint4* bias = reinterpret_cast<uint4*>(sm + L.bias + rr * 128);
             for (int q = 0; q < 8; ++q) bias[q] = make_uint4(0u, 0u, 0u, 0u);
         }
+        if (row < 16) reinterpret_cast<int*>(sm + L.xchg + 4u * kGroups * 128u * 8u)[row] = 0;
         if (!pl.ones_atom || row < 8) {
             uint4* ones = reinterpret_cast<uint4*>(sm + L.ones + row * 128);
             for (int q = 0; q < 8; ++q) ones[q] = make_uint4(0u, 0u, 0u, 0u);
