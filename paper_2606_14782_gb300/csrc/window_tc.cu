@@ -81,16 +81,16 @@ __host__ __device__ inline Smem smem_layout(const Plan& p)
     s.ones = s.k + (uint32_t)p.stages * s.k_stage;
     s.bias = s.ones + (PASS == 2 ? (p.ones_atom ? kOnesAtomBytes : kOnesBytes) : 0u);
     s.xchg = s.bias + (PASS == 2 ? (uint32_t)p.bias_rows * 128u : 0u);
-    // pass 1: partials of groups 1.. per row block; pass 2: every group's
-    // partial sums for four tiles; then per-tile arrival counters / flags
-    s.bars = s.xchg + (PASS == 1 ? (kGroups - 1) * 4u * 128u * 8u : 4u * kGroups * 128u * 8u) + 64u;
+    // every group's partials (pass 1: per row block of a chunk; pass 2: for
+    // four tiles), then the arrival counters
+    s.bars = s.xchg + 4u * kGroups * 128u * 8u + 64u;
     s.bars = (s.bars + 7u) & ~7u;
     s.total = s.bars + 256u;  // barriers, TMEM base, abort flag
     return s;
 }
 
 // Barrier block, 8-byte slots from `base` (a shared-memory address):
-// t_full[4], t_empty[4], q_full, q_empty, drain, ep_all, four spare slots, the
+// t_full[4], t_empty[4], q_full, q_empty, drain, five spare slots, the
 // TMEM base word, the abort word, then k_full[stages], k_empty[stages].
 struct Bars {
     uint32_t base;
@@ -100,7 +100,6 @@ struct Bars {
     __device__ __forceinline__ uint32_t q_full() const { return base + 64u; }
     __device__ __forceinline__ uint32_t q_empty() const { return base + 72u; }
     __device__ __forceinline__ uint32_t drain() const { return base + 80u; }
-    __device__ __forceinline__ uint32_t ep_all() const { return base + 88u; }
     __device__ __forceinline__ uint32_t tmem_slot() const { return base + 128u; }
     __device__ __forceinline__ uint32_t abort() const { return base + 136u; }
     __device__ __forceinline__ uint32_t k_full(int st) const { return base + 144u + 8u * st; }
@@ -116,17 +115,6 @@ __device__ inline Bars bars_at(uint8_t* p, int stages)
     b.base = smem_u32(p);
     b.stages = stages;
     return b;
-}
-
-// Barrier among epilogue warps built on an mbarrier (one arrival per warp),
-// so that it shares the bounded, abort-aware wait of the pipeline.
-__device__ inline bool warp_barrier(uint32_t bar, int& phase, uint32_t abort)
-{
-    __syncwarp();
-    if ((threadIdx.x & 31) == 0) tc::mbar_arrive(bar);
-    const bool ok = tc::mbar_wait(bar, phase & 1, abort);
-    ++phase;
-    return ok;
 }
 
 __device__ inline void raise_abort(const Bars& b, int* err)
@@ -346,13 +334,14 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
     const int quarter = warp & 3;        // TMEM lanes this warp may access
     const int group = (warp - 2) >> 2;   // which 32 tokens of each job
     const uint32_t tmem = tc::ld_shared(b.tmem_slot());
-    float2* xchg = reinterpret_cast<float2*>(sm + L.xchg);  // [group - 1][rb][128]
+    float2* xchg = reinterpret_cast<float2*>(sm + L.xchg);  // [group][rb][128]
+    int* cnt = reinterpret_cast<int*>(xchg + kGroups * 4 * 128);  // arrivals per quarter
     const int nrb = (q_rows + 127) / 128;
     const float c = kLog2e * rsqrtf((float)D);
     const unsigned long long c2 = tc::pack2(c, c);
     int c0, c1;
     chunk_range(a.total_chunks, &c0, &c1);
-    int job = 0, ep_phase = 0;
+    int job = 0;
     bool ok = true;
     for (int g = c0; g < c1 && ok; ++g) {
         const int u = g / a.chunks, ci = g - u * a.chunks;
@@ -412,30 +401,40 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
             }
         }
         if (!ok) break;
-        // merge the groups' statistics of each row, then publish the chunk's partial
-        if (group > 0)
-            for (int rb = 0; rb < nrb; ++rb)
-                xchg[((group - 1) * 4 + rb) * 128 + quarter * 32 + lane] = make_float2(m_run[rb], z_run[rb]);
-        if (!warp_barrier(b.ep_all(), ep_phase, b.abort())) { ok = false; break; }
-        if (group == 0) {
+        // merge the groups' statistics of each row and publish the chunk's
+        // partial: every group leaves its (max, sum) per row block in shared
+        // memory and the last group of this lane quarter to arrive merges
+        // them in group order (no barrier across the epilogue; the groups of
+        // a quarter cannot drift a whole chunk apart, as a TMEM buffer is
+        // only refilled once all of them have read it)
+        for (int rb = 0; rb < nrb; ++rb)
+            xchg[(group * 4 + rb) * 128 + quarter * 32 + lane] = make_float2(m_run[rb], z_run[rb]);
+        __syncwarp();
+        int last = 0;
+        if (lane == 0) {
+            __threadfence_block();
+            last = atomicAdd(cnt + quarter, 1) == kGroups - 1;
+        }
+        last = __shfl_sync(0xffffffffu, last, 0);
+        if (last) {
+            __threadfence_block();
+            const volatile float2* vx = xchg + quarter * 32 + lane;
             for (int rb = 0; rb < nrb; ++rb) {
                 const int r = rb * 128 + quarter * 32 + lane;
-                float M = m_run[rb];
-                for (int gg = 0; gg < kGroups - 1; ++gg)
-                    M = fmaxf(M, xchg[(gg * 4 + rb) * 128 + quarter * 32 + lane].x);
+                float M = -INFINITY;
+                for (int gg = 0; gg < kGroups; ++gg) M = fmaxf(M, vx[(gg * 4 + rb) * 128].x);
                 float Z = 0.f;
-                if (M != -INFINITY) {
-                    Z = z_run[rb] * fast_exp2(m_run[rb] - M);
-                    for (int gg = 0; gg < kGroups - 1; ++gg) {
-                        const float2 o = xchg[(gg * 4 + rb) * 128 + quarter * 32 + lane];
-                        Z += o.y * fast_exp2(o.x - M);
+                if (M != -INFINITY)
+                    for (int gg = 0; gg < kGroups; ++gg) {
+                        const float mz = vx[(gg * 4 + rb) * 128].x, zz = vx[(gg * 4 + rb) * 128].y;
+                        Z = gg == 0 ? zz * fast_exp2(mz - M) : Z + zz * fast_exp2(mz - M);
                     }
-                }
                 if (r < s.rows)
                     a.partial[((size_t)u * a.chunks + ci) * s.rows + r] = make_float2(M, Z);
             }
+            __syncwarp();
+            if (lane == 0) cnt[quarter] = 0;
         }
-        if (!warp_barrier(b.ep_all(), ep_phase, b.abort())) { ok = false; break; }
     }
     if (!ok) raise_abort(b, a.err);
 }
@@ -700,7 +699,6 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, Plan p
         tc::mbar_init(b.q_full(), PASS == 2 ? 2 : 1);  // pass 2: TMA bytes + the bias writes
         tc::mbar_init(b.q_empty(), 1);
         tc::mbar_init(b.drain(), 1);
-        tc::mbar_init(b.ep_all(), kEpiThreads / 32);
         tc::st_shared_volatile(b.abort(), 0u);
         tc::fence_barrier_init();
     }
@@ -708,6 +706,8 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, Plan p
         tc::tmem_alloc(b.tmem_slot(), kTmemCols);
         tc::tmem_relinquish();
     }
+    if (threadIdx.x >= 64 && threadIdx.x < 64 + 16)
+        reinterpret_cast<int*>(sm + L.xchg + 4u * kGroups * 128u * 8u)[threadIdx.x - 64] = 0;
     if (PASS == 2 && threadIdx.x >= 64 && threadIdx.x < 64 + 128) {
         // constant operand: 1 in columns 0-2 of every token row (one atom of
         // 8 rows when ones_atom); the bias operand starts zeroed (the
@@ -717,7 +717,6 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, Plan p
             uint4* bias = reinterpret_cast<uint4*>(sm + L.bias + rr * 128);
             for (int q = 0; q < 8; ++q) bias[q] = make_uint4(0u, 0u, 0u, 0u);
         }
-        if (row < 16) reinterpret_cast<int*>(sm + L.xchg + 4u * kGroups * 128u * 8u)[row] = 0;
         if (!pl.ones_atom || row < 8) {
             uint4* ones = reinterpret_cast<uint4*>(sm + L.ones + row * 128);
             for (int q = 0; q < 8; ++q) ones[q] = make_uint4(0u, 0u, 0u, 0u);
