@@ -45,6 +45,8 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="skip the prefill-normaliser and ablation-sweep measurements")
     return ap.parse_args()
 
 
@@ -334,55 +336,56 @@ def main():
             "gpu_launches": 5 * args.steps, "roofline": roofline, "kernels": kernels,
             "clocks": clocks}
 
-    # the same step when the prefill attention supplies the window rows'
-    # softmax normalisers (no first pass over K)
-    lse = torch.empty((wl.requests, wl.layers, wl.q_heads, wl.window), dtype=torch.float32,
-                      device=dev)
-    pos = torch.arange(wl.seq_len, device=dev)
-    vis = pos[None, :] <= (wl.seq_len - wl.window + torch.arange(wl.window, device=dev))[:, None]
-    for r in range(wl.requests):
-        for l in range(wl.layers):
-            q = x.qwin[r, l].float().view(wl.kv_heads, wl.group, wl.window, wl.head_dim)
-            s_ = torch.einsum("hgwd,hnd->hgwn", q, x.k[r, l].float()) / wl.head_dim ** 0.5
-            lse[r, l] = torch.logsumexp(s_.masked_fill(~vis, float("-inf")), -1).reshape(
-                wl.q_heads, wl.window)
-    del s_
-    for _ in range(3):
-        ctx.compress_with_lse(x.qwin, x.k, x.v, lse, budget, ko, vo, idx)
-    torch.cuda.synchronize()
-    g0 = torch.cuda.Event(enable_timing=True)
-    g1 = torch.cuda.Event(enable_timing=True)
-    g0.record(stream)
-    for _ in range(args.steps):
-        ctx.compress_with_lse(x.qwin, x.k, x.v, lse, budget, ko, vo, idx)
-    g1.record(stream)
-    torch.cuda.synchronize()
-    line["with_prefill_normalisers"] = {
-        "ms_per_step": g0.elapsed_time(g1) / args.steps,
-        "what": "bacon_compress_with_lse: the window rows' softmax normalisers come from the "
-                "prefill attention, so the first pass over K is skipped"}
-    del lse
+    if not args.no_extras:
+        # the same step when the prefill attention supplies the window rows'
+        # softmax normalisers (no first pass over K)
+        lse = torch.empty((wl.requests, wl.layers, wl.q_heads, wl.window), dtype=torch.float32,
+                          device=dev)
+        pos = torch.arange(wl.seq_len, device=dev)
+        vis = pos[None, :] <= (wl.seq_len - wl.window + torch.arange(wl.window, device=dev))[:, None]
+        for r in range(wl.requests):
+            for l in range(wl.layers):
+                q = x.qwin[r, l].float().view(wl.kv_heads, wl.group, wl.window, wl.head_dim)
+                s_ = torch.einsum("hgwd,hnd->hgwn", q, x.k[r, l].float()) / wl.head_dim ** 0.5
+                lse[r, l] = torch.logsumexp(s_.masked_fill(~vis, float("-inf")), -1).reshape(
+                    wl.q_heads, wl.window)
+        del s_
+        for _ in range(3):
+            ctx.compress_with_lse(x.qwin, x.k, x.v, lse, budget, ko, vo, idx)
+        torch.cuda.synchronize()
+        g0 = torch.cuda.Event(enable_timing=True)
+        g1 = torch.cuda.Event(enable_timing=True)
+        g0.record(stream)
+        for _ in range(args.steps):
+            ctx.compress_with_lse(x.qwin, x.k, x.v, lse, budget, ko, vo, idx)
+        g1.record(stream)
+        torch.cuda.synchronize()
+        line["with_prefill_normalisers"] = {
+            "ms_per_step": g0.elapsed_time(g1) / args.steps,
+            "what": "bacon_compress_with_lse: the window rows' softmax normalisers come from the "
+                    "prefill attention, so the first pass over K is skipped"}
+        del lse
 
-    # the paper's ablation / sensitivity grid, every variant selected from
-    # one set of window passes (indices only, no gather)
-    variants = list(workloads.SWEEP_VARIANTS)
-    sidx, slam = ctx.sweep(x.qwin, x.k, budget, variants)
-    for _ in range(3):
-        ctx.sweep(x.qwin, x.k, budget, variants, sidx, slam)
-    torch.cuda.synchronize()
-    g0.record(stream)
-    for _ in range(args.steps):
-        ctx.sweep(x.qwin, x.k, budget, variants, sidx, slam)
-    g1.record(stream)
-    torch.cuda.synchronize()
-    sweep_ms = g0.elapsed_time(g1) / args.steps
-    line["ablation_sweep"] = {
-        "variants": len(variants), "ms_per_sweep": sweep_ms,
-        "ms_per_variant": sweep_ms / len(variants),
-        "separate_whole_steps_ms": len(variants) * ms,
-        "what": "bacon_sweep over the component ablation and the m / r sensitivity grid: "
-                "one set of window passes, then calibration and selection per variant"}
-    del sidx, slam
+        # the paper's ablation / sensitivity grid, every variant selected from
+        # one set of window passes (indices only, no gather)
+        variants = list(workloads.SWEEP_VARIANTS)
+        sidx, slam = ctx.sweep(x.qwin, x.k, budget, variants)
+        for _ in range(3):
+            ctx.sweep(x.qwin, x.k, budget, variants, sidx, slam)
+        torch.cuda.synchronize()
+        g0.record(stream)
+        for _ in range(args.steps):
+            ctx.sweep(x.qwin, x.k, budget, variants, sidx, slam)
+        g1.record(stream)
+        torch.cuda.synchronize()
+        sweep_ms = g0.elapsed_time(g1) / args.steps
+        line["ablation_sweep"] = {
+            "variants": len(variants), "ms_per_sweep": sweep_ms,
+            "ms_per_variant": sweep_ms / len(variants),
+            "separate_whole_steps_ms": len(variants) * ms,
+            "what": "bacon_sweep over the component ablation and the m / r sensitivity grid: "
+                    "one set of window passes, then calibration and selection per variant"}
+        del sidx, slam
 
     # end to end through the host-buffer C call: H2D inputs, compress, D2H outputs
     if not args.no_e2e:
