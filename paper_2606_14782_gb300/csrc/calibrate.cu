@@ -16,7 +16,12 @@ namespace {
 
 using namespace sel;
 
-constexpr int kThreads = 1024;
+// At most kMaxPer tokens per thread.  Threads per CTA depend on the prompt
+// length only (so that every call on the same shape reduces in the same
+// order and gives the same bits): 256 up to 2048 tokens, where several CTAs
+// share an SM, else 1024.
+constexpr int kMaxPer = 24;
+constexpr int kSmallPrompt = 2048;
 
 // Block-wide fp32 sum by a shuffle tree (pairwise, so the rounding error
 // grows with log2 of the count).  FP64 is avoided: its rate on this part is
@@ -150,7 +155,6 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
         else
             for (int i = threadIdx.x; i < N; i += blockDim.x) Vs[i] = Ec[i];
         __syncthreads();
-        constexpr int kMaxPer = 24;  // N <= 24576 with 1024 threads
         float vreg[kMaxPer];
         // persistence: mean of E over the preceding min(m, l) layers (Eqs. 8-9)
 #pragma unroll
@@ -274,7 +278,8 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
     for (int w = threadIdx.x; w < win; w += blockDim.x) out[keep + w] = N - W + w;
 }
 
-__global__ void __launch_bounds__(kThreads)
+template <int T>
+__global__ void __launch_bounds__(T, 1024 / T)
 calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
 {
     const int u = blockIdx.x;
@@ -285,7 +290,8 @@ calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
 // runs unit u under variant v; variant v's indices start v *
 // idx_variant_stride elements after the single-variant layout and its
 // lambdas v * units after a.lambda.
-__global__ void __launch_bounds__(kThreads)
+template <int T>
+__global__ void __launch_bounds__(T, 1024 / T)
 calibrate_sweep_kernel(Shape s, CalibTable t, CalibArgs a)
 {
     const int u = blockIdx.x, v = blockIdx.y;
@@ -297,26 +303,45 @@ calibrate_sweep_kernel(Shape s, CalibTable t, CalibArgs a)
 
 size_t calibrate_smem(int N) { return (size_t)2 * N * sizeof(float); }
 
+namespace {
+
+template <int T>
+cudaError_t launch_select_t(const Shape& s, const Calib& c, const CalibArgs& a, cudaStream_t st)
+{
+    const size_t sm = calibrate_smem(s.N);
+    cudaError_t e = cudaFuncSetAttribute(calibrate_select_kernel<T>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    calibrate_select_kernel<T><<<s.units, T, sm, st>>>(s, c, a);
+    return cudaGetLastError();
+}
+
+template <int T>
+cudaError_t launch_sweep_t(const Shape& s, const CalibTable& t, int variants, const CalibArgs& a,
+                           cudaStream_t st)
+{
+    const size_t sm = calibrate_smem(s.N);
+    cudaError_t e = cudaFuncSetAttribute(calibrate_sweep_kernel<T>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    calibrate_sweep_kernel<T><<<dim3(s.units, variants), T, sm, st>>>(s, t, a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
 cudaError_t launch_calibrate_select(const Shape& s, const Calib& c, const CalibArgs& a,
                                     cudaStream_t st)
 {
-    const size_t sm = calibrate_smem(s.N);
-    cudaError_t e = cudaFuncSetAttribute(calibrate_select_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-    if (e != cudaSuccess) return e;
-    calibrate_select_kernel<<<s.units, kThreads, sm, st>>>(s, c, a);
-    return cudaGetLastError();
+    return s.N <= kSmallPrompt ? launch_select_t<256>(s, c, a, st)
+                               : launch_select_t<1024>(s, c, a, st);
 }
 
 cudaError_t launch_calibrate_sweep(const Shape& s, const CalibTable& t, int variants,
                                    const CalibArgs& a, cudaStream_t st)
 {
-    const size_t sm = calibrate_smem(s.N);
-    cudaError_t e = cudaFuncSetAttribute(calibrate_sweep_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-    if (e != cudaSuccess) return e;
-    calibrate_sweep_kernel<<<dim3(s.units, variants), kThreads, sm, st>>>(s, t, a);
-    return cudaGetLastError();
+    return s.N <= kSmallPrompt ? launch_sweep_t<256>(s, t, variants, a, st)
+                               : launch_sweep_t<1024>(s, t, variants, a, st);
 }
 
 }  // namespace bacon

@@ -39,7 +39,7 @@ constexpr int kSelBins = 1 << kSelBits;
 // the data's own range, so few keys share one), takes the bin where the
 // count from the top reaches k, and narrows the range to it, until a bin is
 // one key.  At most three passes for 32-bit keys.  Every thread returns the
-// same result; blockDim.x must be 1024 (32 warps x 64 bins in the scan).
+// same result; blockDim.x must be a power of two from 64 to 1024.
 // kmin / kmax: this thread's share of the key range (the callers that know
 // it from an earlier pass over the keys pass it in; see radix_select_by).
 template <typename KeyFn>
@@ -83,22 +83,25 @@ __device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist
             }
         }
         __syncthreads();
-        // bins from the top: lane l of warp w holds bins 64 w + 63 - 2 l and
-        // 64 w + 62 - 2 l; warp totals first, then the boundary warp's bins
-        const int bhi = 64 * warp + 63 - 2 * lane;
-        const int chi = hist[bhi], clo = hist[bhi - 1];
-        int incl = chi + clo;
+        // bins from the top: warp w holds the w-th slice of bpw bins and its
+        // lane l the bpl bins just below the top l bpl of that slice; warp
+        // totals first, then the boundary warp's lanes, then the lane's bins
+        const int nwarps = (int)(blockDim.x >> 5);
+        const int bpw = kSelBins / nwarps, bpl = bpw / 32;
+        const int ltop = bpw * (warp + 1) - 1 - bpl * lane;  // this lane's highest bin
+        int mine = 0;
+        for (int q = 0; q < bpl; ++q) mine += hist[ltop - q];
+        int incl = mine;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
             const int y = __shfl_up_sync(0xffffffffu, incl, o);
             if (lane >= o) incl += y;
         }
-        __syncthreads();  // everyone has read the bins
         if (lane == 31) hist[kSelBins + warp] = incl;  // warp total
         __syncthreads();
         if (warp == 0) {
-            // warps from the top: above[w] = totals of warps w + 1 .. 31
-            const int tot = hist[kSelBins + 31 - lane];
+            // warps from the top: above[w] = totals of warps w + 1 .. nwarps - 1
+            const int tot = lane < nwarps ? hist[kSelBins + nwarps - 1 - lane] : 0;
             int cum = tot;
 #pragma unroll
             for (int o = 1; o < 32; o <<= 1) {
@@ -106,10 +109,10 @@ __device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist
                 if (lane >= o) cum += y;
             }
             const uint32_t hit = __ballot_sync(0xffffffffu, cum >= remaining);
-            const int first = __ffs(hit) - 1;  // the boundary warp is 31 - first
+            const int first = __ffs(hit) - 1;  // the boundary warp is nwarps - 1 - first
             const int above = __shfl_sync(0xffffffffu, cum - tot, first);
             if (lane == 0) {
-                bcast[2] = 31 - first;
+                bcast[2] = nwarps - 1 - first;
                 bcast[3] = above;
             }
         }
@@ -119,15 +122,16 @@ __device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist
             const uint32_t hit = __ballot_sync(0xffffffffu, incl >= rem);
             const int first = __ffs(hit) - 1;
             if (lane == first) {
-                const int before = incl - chi - clo;  // bins above this lane's pair
-                if (before + chi >= rem) {
-                    bcast[0] = bhi;
-                    bcast[1] = rem - before;
-                    bcast[4] = chi;
-                } else {
-                    bcast[0] = bhi - 1;
-                    bcast[1] = rem - before - chi;
-                    bcast[4] = clo;
+                int before = incl - mine;  // bins above this lane's
+                for (int q = 0; q < bpl; ++q) {
+                    const int c = hist[ltop - q];
+                    if (before + c >= rem) {
+                        bcast[0] = ltop - q;
+                        bcast[1] = rem - before;
+                        bcast[4] = c;
+                        break;
+                    }
+                    before += c;
                 }
             }
         }
