@@ -410,12 +410,17 @@ def main():
             ctx.compress_host(hq, hk, hv, budget, hko, hvo, hidx)
         torch.cuda.synchronize()
         e2e_ms = reduce_step_time((time.perf_counter() - t0) * 1e3 / args.e2e_steps, world, dev)
-        h2d = sum(t.numel() * t.element_size() for t in (hq, hk, hv))
+        # page-locked values are not uploaded: the gather reads the kept rows
+        # in place (the library's host path), so only those rows cross
+        v_rows = units * kept * wl.head_dim * hv.element_size()
+        h2d = sum(t.numel() * t.element_size() for t in (hq, hk)) + (
+            v_rows if hv.is_pinned() else hv.numel() * hv.element_size())
         d2h = sum(t.numel() * t.element_size() for t in (hko, hvo, hidx))
         line["e2e"] = {"value": job_throughput(units, world, e2e_ms), "unit": UNIT,
                        "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d,
                        "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
-                       "path": "bacon_compress_host (pinned host buffers)"}
+                       "path": "bacon_compress_host (pinned host buffers; queries and keys "
+                               "uploaded, kept value rows read in place)"}
     ctx.close()
 
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -248,7 +248,10 @@ void bacon_pyramid_budgets(int layers, int window, int budget, int beta, int* ou
  *   q_win [requests][layers][Hq][W][d], k, v [requests][layers][Hkv][N][d],
  *   k_out, v_out [requests][layers][Hkv][kept][d],
  *   idx_out [requests][layers][Hkv][kept].
- * Page-locked host memory gives the full copy bandwidth. */
+ * Page-locked host memory gives the full copy bandwidth.  When `v` is
+ * page-locked memory the device can address (allocated or registered
+ * through CUDA, 16-byte aligned), it is not uploaded: the gather reads only
+ * the kept rows from it in place. */
 bacon_status bacon_compress_host(bacon_ctx* ctx, int requests,
                                  const void* q_win, const void* k,
                                  const void* v, int seq_len, int budget,

@@ -97,7 +97,7 @@ struct bacon_ctx {
     void* hko_buf = nullptr;
     void* hvo_buf = nullptr;
     int32_t* hidx_buf = nullptr;
-    size_t hq_cap = 0, hkv_cap = 0, hout_cap = 0, hidx_cap = 0;
+    size_t hq_cap = 0, hk_cap = 0, hv_cap = 0, hko_cap = 0, hvo_cap = 0, hidx_cap = 0;
     // TMA descriptors of the last whole-step call: [kMaxPairs] K maps, then
     // [kMaxPairs] window-query maps (device copy + pinned host staging)
     CUtensorMap* d_maps = nullptr;
@@ -453,6 +453,20 @@ bacon_status sweep_device(bacon_ctx* c, int R, const void* const* q, const void*
     prof.commit();
     c->last_units = 0;  // S, V, B~ and lambda of the scratch are not this call's
     return BACON_OK;
+}
+
+// Device address of page-locked host memory the current device can read
+// (registered or allocated through CUDA, 16-byte aligned), else null.
+const void* host_device_pointer(const void* p)
+{
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    if (at.type != cudaMemoryTypeHost || !at.devicePointer || !aligned16(at.devicePointer))
+        return nullptr;
+    return at.devicePointer;
 }
 
 bacon_status check_pointer_arrays(const bacon_ctx* c, int pairs, const void* const* q,
@@ -932,16 +946,19 @@ bacon_status bacon_compress_host(bacon_ctx* ctx, int requests, const void* q_win
     const size_t o_pair = (size_t)ctx->hkv * kept * ctx->d;
     const size_t idx_count = (size_t)pairs * ctx->hkv * kept;
     if ((rc = grow(&ctx->hq_buf, &ctx->hq_cap, q_pair * pairs * 2, "queries")) != BACON_OK) return rc;
-    size_t kv_cap = ctx->hkv_cap;
-    if ((rc = grow(&ctx->hk_buf, &kv_cap, kv_pair * pairs * 2, "keys")) != BACON_OK) return rc;
-    kv_cap = ctx->hkv_cap;
-    if ((rc = grow(&ctx->hv_buf, &kv_cap, kv_pair * pairs * 2, "values")) != BACON_OK) return rc;
-    ctx->hkv_cap = kv_cap;
-    size_t o_cap = ctx->hout_cap;
-    if ((rc = grow(&ctx->hko_buf, &o_cap, o_pair * pairs * 2, "compacted keys")) != BACON_OK) return rc;
-    o_cap = ctx->hout_cap;
-    if ((rc = grow(&ctx->hvo_buf, &o_cap, o_pair * pairs * 2, "compacted values")) != BACON_OK) return rc;
-    ctx->hout_cap = o_cap;
+    // Values are only read where a row is kept (about budget / seq_len of
+    // them): when the caller's value buffer is page-locked host memory the
+    // device can address, the gather reads those rows in place instead of
+    // uploading the whole tensor.
+    const void* v_dev = host_device_pointer(v);
+    if ((rc = grow(&ctx->hk_buf, &ctx->hk_cap, kv_pair * pairs * 2, "keys")) != BACON_OK) return rc;
+    if (!v_dev &&
+        (rc = grow(&ctx->hv_buf, &ctx->hv_cap, kv_pair * pairs * 2, "values")) != BACON_OK)
+        return rc;
+    if ((rc = grow(&ctx->hko_buf, &ctx->hko_cap, o_pair * pairs * 2, "compacted keys")) != BACON_OK)
+        return rc;
+    if ((rc = grow(&ctx->hvo_buf, &ctx->hvo_cap, o_pair * pairs * 2, "compacted values")) != BACON_OK)
+        return rc;
     if ((rc = grow(&ctx->hidx_buf, &ctx->hidx_cap, idx_count * 4, "indices")) != BACON_OK) return rc;
 
     if (!ctx->h2d) {
@@ -971,8 +988,9 @@ bacon_status bacon_compress_host(bacon_ctx* ctx, int requests, const void* q_win
                                    cudaMemcpyHostToDevice, ctx->h2d), "query upload");
         BACON_CUDA(cudaMemcpyAsync(static_cast<char*>(ctx->hk_buf) + r * kb, kh + r * kb, kb,
                                    cudaMemcpyHostToDevice, ctx->h2d), "key upload");
-        BACON_CUDA(cudaMemcpyAsync(static_cast<char*>(ctx->hv_buf) + r * kb, vh + r * kb, kb,
-                                   cudaMemcpyHostToDevice, ctx->h2d), "value upload");
+        if (!v_dev)
+            BACON_CUDA(cudaMemcpyAsync(static_cast<char*>(ctx->hv_buf) + r * kb, vh + r * kb, kb,
+                                       cudaMemcpyHostToDevice, ctx->h2d), "value upload");
         BACON_CUDA(cudaEventRecord(ctx->ev_in[r], ctx->h2d), "event");
     }
 
@@ -984,7 +1002,7 @@ bacon_status bacon_compress_host(bacon_ctx* ctx, int requests, const void* q_win
     for (int i = 0; i < pairs; ++i) {
         qs[i] = static_cast<const uint16_t*>(ctx->hq_buf) + q_pair * i;
         ks[i] = static_cast<const uint16_t*>(ctx->hk_buf) + kv_pair * i;
-        vs[i] = static_cast<const uint16_t*>(ctx->hv_buf) + kv_pair * i;
+        vs[i] = static_cast<const uint16_t*>(v_dev ? v_dev : ctx->hv_buf) + kv_pair * i;
         kos[i] = static_cast<uint16_t*>(ctx->hko_buf) + o_pair * i;
         vos[i] = static_cast<uint16_t*>(ctx->hvo_buf) + o_pair * i;
     }

@@ -242,7 +242,9 @@ def test_layer_path_matches_whole_step():
     ctx.close()
 
 
-def test_host_path_matches_device_path():
+@pytest.mark.parametrize("pinned", ["all", "none", "values_pageable"])
+def test_host_path_matches_device_path(pinned):
+    """Page-locked values are gathered in place, pageable ones uploaded."""
     wl = workloads.CONFIGS["tiny"].with_(requests=2, layers=3, seq_len=700, visual=(16, 650))
     x = workloads.generate(wl, seed=4, device="cuda")
     budget = 80
@@ -250,13 +252,21 @@ def test_host_path_matches_device_path():
     p = bacon.default_params(max_seq_len=wl.seq_len, max_requests=2)
     ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool,
                         budget, params=p)
-    qh, kh, vh = (t.cpu().pin_memory() for t in (x.qwin, x.k, x.v))
+    qh, kh, vh = (t.cpu() for t in (x.qwin, x.k, x.v))
+    if pinned == "all":
+        qh, kh, vh = (t.pin_memory() for t in (qh, kh, vh))
+    elif pinned == "values_pageable":
+        qh, kh = qh.pin_memory(), kh.pin_memory()
     ko, vo, idx = ctx.compress_host(qh, kh, vh, budget)
     assert np.array_equal(idx.numpy(), dev["idx"])
     assert torch.equal(ko, dev["Kc"]) and torch.equal(vo, dev["Vc"])
     # a second call reuses the staging buffers
     ko2, _, idx2 = ctx.compress_host(qh, kh, vh, budget)
     assert torch.equal(ko2, ko) and torch.equal(idx2, idx)
+    # switching between in-place and uploaded values on one context
+    other = vh.pin_memory() if not vh.is_pinned() else vh.clone()
+    _, vo3, idx3 = ctx.compress_host(qh, kh, other, budget)
+    assert torch.equal(vo3, dev["Vc"]) and np.array_equal(idx3.numpy(), dev["idx"])
     ctx.close()
 
 
