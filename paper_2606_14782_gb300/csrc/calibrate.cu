@@ -104,7 +104,7 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
     const int N = s.N, W = s.W;
     float* Sb = sm;      // pooled backbone B~, then the final score S
     float* Vs = sm + N;  // calibrated evidence V
-    __shared__ int hist[kSelBins + 32];
+    __shared__ int hist[kSelHist];
     __shared__ int bcast[8];
     __shared__ int warp_sums[32];
     __shared__ float red[4 * 33];

@@ -28,9 +28,13 @@ struct SelectResult {
     __device__ __forceinline__ bool all_ties_in() const { return need == count_eq; }
 };
 
-// Histogram bins of one select pass (shared memory of the caller).
+// Histogram bins of one select pass; the caller's shared array `hist` holds
+// kSelHist ints: the bins, 32 warp totals, a counter and a buffer of up to
+// kSelCap keys.
 constexpr int kSelBits = 11;
 constexpr int kSelBins = 1 << kSelBits;
+constexpr int kSelCap = 2048;
+constexpr int kSelHist = kSelBins + 64 + kSelCap;
 
 // k-th best key over the included elements of [0, n) (1 <= k <= their
 // count).  First the range [kmin, kmax] of the included keys, then passes
@@ -69,20 +73,37 @@ __device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist
     while (((span - 1u) >> shift) >= (uint64_t)kSelBins) ++shift;  // top bin index < kSelBins
     uint64_t width = span;  // keys of the current range: [lo, lo + width)
     int remaining = k;
+    // Once the current range holds at most kSelCap keys, the next pass also
+    // copies them into the buffer and the passes after it read only that.
+    int* bufcnt = hist + kSelBins + 32;
+    uint32_t* buf = reinterpret_cast<uint32_t*>(hist + kSelBins + 64);
+    int in_range = -1, nbuf = -1;  // unknown / not compacted
     __syncthreads();
     while (true) {
         for (int b = threadIdx.x; b < kSelBins; b += blockDim.x) hist[b] = 0;
+        const bool collect = nbuf < 0 && in_range >= 0 && in_range <= kSelCap;
+        if (threadIdx.x == 0) *bufcnt = 0;
         __syncthreads();
-        for (int i0 = threadIdx.x; i0 < n; i0 += 4 * blockDim.x) {
+        if (nbuf >= 0) {
+            for (int i = threadIdx.x; i < nbuf; i += blockDim.x) {
+                const uint32_t key = buf[i];
+                if (key >= lo && (uint64_t)(key - lo) < width) atomicAdd(&hist[(key - lo) >> shift], 1);
+            }
+        } else {
+            for (int i0 = threadIdx.x; i0 < n; i0 += 4 * blockDim.x) {
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int i = i0 + q * (int)blockDim.x;
-                uint32_t key = 0u;
-                if (i < n && key_of(i, key) && key >= lo && (uint64_t)(key - lo) < width)
-                    atomicAdd(&hist[(key - lo) >> shift], 1);
+                for (int q = 0; q < 4; ++q) {
+                    const int i = i0 + q * (int)blockDim.x;
+                    uint32_t key = 0u;
+                    if (i < n && key_of(i, key) && key >= lo && (uint64_t)(key - lo) < width) {
+                        atomicAdd(&hist[(key - lo) >> shift], 1);
+                        if (collect) buf[atomicAdd(bufcnt, 1)] = key;
+                    }
+                }
             }
         }
         __syncthreads();
+        if (collect) nbuf = *bufcnt;
         // bins from the top: warp w holds the w-th slice of bpw bins and its
         // lane l the bpl bins just below the top l bpl of that slice; warp
         // totals first, then the boundary warp's lanes, then the lane's bins
@@ -139,6 +160,7 @@ __device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist
         lo += (uint32_t)bcast[0] << shift;
         remaining = bcast[1];
         const int in_bin = bcast[4];
+        in_range = in_bin;
         width = (uint64_t)1 << shift;
         __syncthreads();
         if (shift == 0) return {lo, remaining, in_bin};
