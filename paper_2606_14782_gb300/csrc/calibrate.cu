@@ -6,8 +6,11 @@
 //   S = B~ + lambda V                                 (Eq. 16)
 //   the K best candidates by S, ascending, then the window (Eq. 17)
 // Both "best k" sets use one order: larger value first, equal values ->
-// lower position first (select.cuh: radix select, then index-ordered
-// warp-segmented sweeps that resolve ties and emit ascending positions).
+// lower position first (select.cuh: range-adaptive radix select, then
+// index-ordered warp-segmented sweeps that resolve ties and emit ascending
+// positions).  The two standard deviations come from one sweep that sums
+// moments about fixed shifts in fp32 (the shifts keep the differences
+// small, so no precision is lost to cancellation).
 #include "common.cuh"
 #include "select.cuh"
 

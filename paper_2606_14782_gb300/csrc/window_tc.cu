@@ -1,25 +1,28 @@
 // Window scores (Eqs. 1, 2, 4) on the 5th-generation tensor cores.
 //
-// Same two-pass structure as the softmax needs (see window.cu), built for
-// sm_103a:
+// A softmax row must be normalised over all N keys before any B_i is final,
+// so K is streamed twice, by two persistent kernels built for sm_103a:
 //   * K tiles (128 tokens x d) and the kv-head's G*W window rows are brought
 //     into shared memory by TMA in the 128-byte-swizzled K-major layout that
 //     tcgen05.mma reads directly;
 //   * one thread issues tcgen05.mma (bf16 x bf16 -> fp32) into TMEM; the
 //     accumulators never visit registers until the epilogue reads them;
 //   * sixteen epilogue warps (four groups, each with one warp per TMEM lane
-//     quarter) share every job's columns and turn logits into softmax
-//     statistics (pass 1) or per-token sums (pass 2) while the MMA of the
-//     next job runs into another TMEM buffer; exp2 runs on the SFU.
-// Pass 1 (stats):  D[row][token], 128 rows x 128 tokens per job, 4 TMEM
-//                  buffers; a thread owns one window row and 32 tokens.
-// Pass 2 (scores): D[token][row], 128 tokens x up to 128 rows per job, 4
-//                  TMEM buffers (so the next tile's MMA overlaps this tile's
-//                  epilogue); a thread owns one token and every fourth
-//                  16-row piece of the tile.
-// Each CTA is persistent and takes a contiguous range of 1024-token chunks
-// of the flattened (unit, chunk) space, so a CTA reloads the window rows only
-// when its range crosses into the next (request, layer, kv-head).
+//     quarter) turn logits into softmax statistics (pass 1) or per-token
+//     sums (pass 2) while the MMA of the next job runs into another TMEM
+//     accumulator; exp2 runs on the SFU.
+// Pass 1 (stats):  D[row][token], 128 rows x 128 tokens per job, four
+//                  128-column accumulators; a thread owns one window row and
+//                  32 tokens of every job.
+// Pass 2 (scores): D[token][row], 128 tokens x up to 256 rows per job, two
+//                  256-column accumulators (four of 128 when shared memory
+//                  is short); the accumulator starts from each row's
+//                  -lse2 / c (one extra MMA against a constant operand) and
+//                  a thread owns one token and 32-column slices of a job.
+// Each CTA takes a contiguous range of 1024-token chunks of the flattened
+// (unit, chunk) space, so it reloads the window rows only when its range
+// crosses into the next (request, layer, kv-head).  The epilogue groups meet
+// through shared-memory slots and arrival counters, never at a barrier.
 // Every wait is bounded: on timeout the CTA raises an abort flag, records
 // kErrTimeout in the error word, drains its own copies and MMAs, frees TMEM
 // and returns.
