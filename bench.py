@@ -125,16 +125,27 @@ class ClockSampler:
 
 # --------------------------------------------------------- traffic
 
+def source_digest(names) -> str:
+    """sha256[:16] of the named csrc files with comments and blank space
+    removed, so that editing a comment does not void a measurement."""
+    import re
+    h = hashlib.sha256()
+    for name in names:
+        text = open(os.path.join(ROOT, "paper_2606_14782_gb300", "csrc", name)).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", "", text)
+        h.update("".join(text.split()).encode())
+    return h.hexdigest()[:16]
+
+
 def kernel_traffic(kernel: str):
     """DRAM bytes per launch from the committed ncu summary, or None when the
-    kernel's source changed since the counters were taken."""
+    kernel's sources changed since the counters were taken."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
             rec = json.load(f)[kernel]
-        src = os.path.join(ROOT, "paper_2606_14782_gb300", "csrc", rec["source"])
-        digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-        if digest != rec["source_sha256_16"]:
+        if source_digest(rec["sources"]) != rec["code_sha256_16"]:
             return None
         return float(rec["dram_bytes_per_launch"])
     except Exception:
