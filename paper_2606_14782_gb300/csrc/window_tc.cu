@@ -84,17 +84,18 @@ __host__ __device__ inline Smem smem_layout(const Plan& p)
     s.ones = s.k + (uint32_t)p.stages * s.k_stage;
     s.bias = s.ones + (PASS == 2 ? (p.ones_atom ? kOnesAtomBytes : kOnesBytes) : 0u);
     s.xchg = s.bias + (PASS == 2 ? (uint32_t)p.bias_rows * 128u : 0u);
-    // every group's partials (pass 1: per row block of a chunk; pass 2: for
-    // four tiles), then the arrival counters
-    s.bars = s.xchg + 4u * kGroups * 128u * 8u + 64u;
+    // every group's partials: pass 1 per row block of a chunk, pass 2 for
+    // two tiles
+    s.bars = s.xchg + (PASS == 1 ? 4u : 2u) * kGroups * 128u * 8u;
     s.bars = (s.bars + 7u) & ~7u;
-    s.total = s.bars + 256u;  // barriers, TMEM base, abort flag
+    s.total = s.bars + 144u + 8u * (2u * (uint32_t)p.stages + 16u);  // barriers, TMEM base, abort flag
     return s;
 }
 
 // Barrier block, 8-byte slots from `base` (a shared-memory address):
 // t_full[4], t_empty[4], q_full, q_empty, drain, five spare slots, the
-// TMEM base word, the abort word, then k_full[stages], k_empty[stages].
+// TMEM base word, the abort word, then k_full[stages], k_empty[stages],
+// x_full[2][4], x_empty[2][4].
 struct Bars {
     uint32_t base;
     int stages;
@@ -109,6 +110,16 @@ struct Bars {
     __device__ __forceinline__ uint32_t k_empty(int st) const
     {
         return base + 144u + 8u * (stages + st);
+    }
+    // pass 2, exchange slot p (tile parity) of lane quarter q: the three
+    // non-merging groups' partial sums are in it / the merging group has read it
+    __device__ __forceinline__ uint32_t x_full(int p, int q) const
+    {
+        return base + 144u + 8u * (2 * stages + 4 * p + q);
+    }
+    __device__ __forceinline__ uint32_t x_empty(int p, int q) const
+    {
+        return base + 144u + 8u * (2 * stages + 8 + 4 * p + q);
     }
 };
 
@@ -338,13 +349,12 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
     const int group = (warp - 2) >> 2;   // which 32 tokens of each job
     const uint32_t tmem = tc::ld_shared(b.tmem_slot());
     float2* xchg = reinterpret_cast<float2*>(sm + L.xchg);  // [group][rb][128]
-    int* cnt = reinterpret_cast<int*>(xchg + kGroups * 4 * 128);  // arrivals per quarter
     const int nrb = (q_rows + 127) / 128;
     const float c = kLog2e * rsqrtf((float)D);
     const unsigned long long c2 = tc::pack2(c, c);
     int c0, c1;
     chunk_range(a.total_chunks, &c0, &c1);
-    int job = 0;
+    int job = 0, nch = 0;
     bool ok = true;
     for (int g = c0; g < c1 && ok; ++g) {
         const int u = g / a.chunks, ci = g - u * a.chunks;
@@ -398,45 +408,66 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
                         acc[(j >> 1) & 3] = tc::add2(acc[(j >> 1) & 3], tc::pack2(fast_exp2(tt.x), fast_exp2(tt.y)));
                     }
                     const float2 s2 = tc::unpack2(tc::add2(tc::add2(acc[0], acc[1]), tc::add2(acc[2], acc[3])));
-                    z_run[rb] = z_run[rb] * fast_exp2(m_run[rb] - m_new) + (s2.x + s2.y);
-                    m_run[rb] = m_new;
+                    const float zs = s2.x + s2.y;
+                    if (m_new > m_run[rb]) {
+                        z_run[rb] = z_run[rb] * fast_exp2(m_run[rb] - m_new) + zs;
+                        m_run[rb] = m_new;
+                    } else {
+                        z_run[rb] += zs;
+                    }
                 }
             }
         }
         if (!ok) break;
         // merge the groups' statistics of each row and publish the chunk's
-        // partial: every group leaves its (max, sum) per row block in shared
-        // memory and the last group of this lane quarter to arrive merges
-        // them in group order (no barrier across the epilogue; the groups of
-        // a quarter cannot drift a whole chunk apart, as a TMEM buffer is
-        // only refilled once all of them have read it)
-        for (int rb = 0; rb < nrb; ++rb)
-            xchg[(group * 4 + rb) * 128 + quarter * 32 + lane] = make_float2(m_run[rb], z_run[rb]);
-        __syncwarp();
-        int last = 0;
-        if (lane == 0) {
-            __threadfence_block();
-            last = atomicAdd(cnt + quarter, 1) == kGroups - 1;
-        }
-        last = __shfl_sync(0xffffffffu, last, 0);
-        if (last) {
-            __threadfence_block();
-            const volatile float2* vx = xchg + quarter * 32 + lane;
-            for (int rb = 0; rb < nrb; ++rb) {
-                const int r = rb * 128 + quarter * 32 + lane;
-                float M = -INFINITY;
-                for (int gg = 0; gg < kGroups; ++gg) M = fmaxf(M, vx[(gg * 4 + rb) * 128].x);
-                float Z = 0.f;
-                if (M != -INFINITY)
-                    for (int gg = 0; gg < kGroups; ++gg) {
-                        const float mz = vx[(gg * 4 + rb) * 128].x, zz = vx[(gg * 4 + rb) * 128].y;
-                        Z = gg == 0 ? zz * fast_exp2(mz - M) : Z + zz * fast_exp2(mz - M);
-                    }
-                if (r < s.rows)
-                    a.partial[((size_t)u * a.chunks + ci) * s.rows + r] = make_float2(M, Z);
+        // partial: group n mod 4 of this CTA's n-th chunk waits until the
+        // other three groups of its lane quarter have left their (max, sum)
+        // per row block in shared memory, merges them in group order and
+        // frees the slot for the next chunk
+        const int merger = nch & 3;
+        const uint32_t ph = (uint32_t)nch & 1u;
+        ++nch;
+        if (group != merger) {
+            if (!tc::mbar_wait(b.x_empty(0, quarter), ph ^ 1u, b.abort())) {
+                ok = false;
+                break;
+            }
+#pragma unroll
+            for (int rb = 0; rb < 4; ++rb) {
+                if (rb >= nrb) break;
+                xchg[(group * 4 + rb) * 128 + quarter * 32 + lane] = make_float2(m_run[rb], z_run[rb]);
             }
             __syncwarp();
-            if (lane == 0) cnt[quarter] = 0;
+            if (lane == 0) tc::mbar_arrive(b.x_full(0, quarter));
+        } else {
+            if (!tc::mbar_wait(b.x_full(0, quarter), ph, b.abort())) {
+                ok = false;
+                break;
+            }
+            const float2* vx = xchg + quarter * 32 + lane;
+#pragma unroll
+            for (int rb = 0; rb < 4; ++rb) {
+                if (rb >= nrb) break;
+                float2 mz[kGroups];
+#pragma unroll
+                for (int gg = 0; gg < kGroups; ++gg)
+                    mz[gg] = gg == group ? make_float2(m_run[rb], z_run[rb]) : vx[(gg * 4 + rb) * 128];
+                float M = -INFINITY;
+#pragma unroll
+                for (int gg = 0; gg < kGroups; ++gg) M = fmaxf(M, mz[gg].x);
+                float Z = 0.f;
+                if (M != -INFINITY) {
+#pragma unroll
+                    for (int gg = 0; gg < kGroups; ++gg) {
+                        const float zz = mz[gg].y * fast_exp2(mz[gg].x - M);
+                        Z = gg == 0 ? zz : Z + zz;
+                    }
+                }
+                const int r = rb * 128 + quarter * 32 + lane;
+                if (r < s.rows) a.partial[((size_t)u * a.chunks + ci) * s.rows + r] = make_float2(M, Z);
+            }
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(b.x_empty(0, quarter));
         }
     }
     if (!ok) raise_abort(b, a.err);
@@ -577,8 +608,7 @@ __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, 
     const int quarter = warp & 3;
     const int group = (warp - 2) >> 2;
     const uint32_t tl = tc::ld_shared(b.tmem_slot()) + ((uint32_t)(quarter * 32) << 16);
-    float2* xs = reinterpret_cast<float2*>(sm + L.xchg);  // [4][kGroups][128]
-    int* cnt = reinterpret_cast<int*>(xs + 4 * kGroups * 128);  // [4 tiles][4 quarters]
+    float2* xs = reinterpret_cast<float2*>(sm + L.xchg);  // [2][kGroups][128]
     ScoreCtx k;
     const float c = kLog2e * rsqrtf((float)D);
     k.c2 = tc::pack2(c, c);
@@ -589,7 +619,7 @@ __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, 
         if (16 * g + 15 < s.rows && (16 * g + 15) % s.W == s.W - 1) k.qmask |= 1u << g;
     int c0, c1;
     chunk_range(a.total_chunks, &c0, &c1);
-    int job = 0;
+    int job = 0, ntile = 0;
     bool ok = true;
     for (int g = c0; g < c1 && ok; ++g) {
         const int u = g / a.chunks, ci = g - u * a.chunks;
@@ -604,38 +634,46 @@ __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, 
                      : score_tile<FASTQ, false, NBUF_LOG2>(jt, job, group, tl, b, k, tok, bacc, qacc);
             if (!ok) break;
             const float2 b2 = tc::unpack2(tc::add2(bacc[0], bacc[1]));
-            float bsum = b2.x + b2.y;
-            float qsum = qacc * (float)s.W;
-            // the groups' partial sums of a token meet in shared memory,
-            // four tile slots deep; the last group to arrive adds them in
-            // group order and stores the token's B, Q and E
-            float2* slot = xs + (size_t)((t & 3) * kGroups) * 128 + quarter * 32 + lane;
-            slot[group * 128] = make_float2(bsum, qsum);
-            __syncwarp();
-            int last = 0;
-            if (lane == 0) {
-                __threadfence_block();
-                last = atomicAdd(cnt + (t & 3) * 4 + quarter, 1) == kGroups - 1;
-            }
-            last = __shfl_sync(0xffffffffu, last, 0);
-            if (last) {
-                __threadfence_block();
-                const volatile float2* vs = slot;
-                float2 o = make_float2(vs[0].x, vs[0].y);
-                bsum = o.x;
-                qsum = o.y;
-                for (int gg = 1; gg < kGroups; ++gg) {
-                    bsum += vs[gg * 128].x;
-                    qsum += vs[gg * 128].y;
+            const float bsum = b2.x + b2.y;
+            const float qsum = qacc * (float)s.W;
+            // the groups' partial sums of a token meet in shared memory (two
+            // slots, used by this CTA's tiles in turn); group n mod 4 of the
+            // CTA's n-th tile adds them in group order once the other three
+            // have arrived on the slot's barrier, frees the slot and stores
+            // the token's B, Q and E
+            const int par = ntile & 1;
+            const uint32_t ph = (uint32_t)(ntile >> 1) & 1u;
+            const int merger = ntile & 3;
+            ++ntile;
+            float2* slot = xs + (size_t)(par * kGroups) * 128 + quarter * 32 + lane;
+            if (group != merger) {
+                if (!tc::mbar_wait(b.x_empty(par, quarter), ph ^ 1u, b.abort())) {
+                    ok = false;
+                    break;
                 }
-                if (tok < s.N) {
-                    const size_t idx = (size_t)u * s.N + tok;
-                    a.B[idx] = bsum;
-                    a.Q[idx] = qsum;
-                    a.E[idx] = fmaxf(qsum - bsum, 0.f);
+                slot[group * 128] = make_float2(bsum, qsum);
+                __syncwarp();
+                if (lane == 0) tc::mbar_arrive(b.x_full(par, quarter));
+            } else {
+                if (!tc::mbar_wait(b.x_full(par, quarter), ph, b.abort())) {
+                    ok = false;
+                    break;
+                }
+                float bt = 0.f, qt = 0.f;
+#pragma unroll
+                for (int gg = 0; gg < kGroups; ++gg) {
+                    const float2 o = gg == group ? make_float2(bsum, qsum) : slot[gg * 128];
+                    bt = gg == 0 ? o.x : bt + o.x;
+                    qt = gg == 0 ? o.y : qt + o.y;
                 }
                 __syncwarp();
-                if (lane == 0) cnt[(t & 3) * 4 + quarter] = 0;
+                if (lane == 0) tc::mbar_arrive(b.x_empty(par, quarter));
+                if (tok < s.N) {
+                    const size_t idx = (size_t)u * s.N + tok;
+                    a.B[idx] = bt;
+                    a.Q[idx] = qt;
+                    a.E[idx] = fmaxf(qt - bt, 0.f);
+                }
             }
         }
     }
@@ -702,6 +740,10 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, Plan p
         tc::mbar_init(b.q_full(), PASS == 2 ? 2 : 1);  // pass 2: TMA bytes + the bias writes
         tc::mbar_init(b.q_empty(), 1);
         tc::mbar_init(b.drain(), 1);
+        for (int i = 0; i < 8; ++i) {
+            tc::mbar_init(b.x_full(i >> 2, i & 3), kGroups - 1);
+            tc::mbar_init(b.x_empty(i >> 2, i & 3), 1);
+        }
         tc::st_shared_volatile(b.abort(), 0u);
         tc::fence_barrier_init();
     }
@@ -709,8 +751,6 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, Plan p
         tc::tmem_alloc(b.tmem_slot(), kTmemCols);
         tc::tmem_relinquish();
     }
-    if (threadIdx.x >= 64 && threadIdx.x < 64 + 16)
-        reinterpret_cast<int*>(sm + L.xchg + 4u * kGroups * 128u * 8u)[threadIdx.x - 64] = 0;
     if (PASS == 2 && threadIdx.x >= 64 && threadIdx.x < 64 + 128) {
         // constant operand: 1 in columns 0-2 of every token row (one atom of
         // 8 rows when ones_atom); the bias operand starts zeroed (the

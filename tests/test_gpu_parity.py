@@ -161,6 +161,10 @@ EDGE = [
     ("pool1_rho3", dict(seq_len=640), 64, dict(rho=3)),
     ("two_requests", dict(seq_len=513, requests=2, visual=(16, 480)), 80, {}),
     ("long_tail_chunks", dict(seq_len=3000, layers=2, visual=(16, 2900)), 200, {}),
+    # more chunks than SMs, units of 9 tiles: each CTA's range of chunks
+    # crosses unit boundaries with an odd number of tiles per unit
+    ("odd_tiles_many_units", dict(seq_len=1152, layers=24, q_heads=8, kv_heads=8,
+                                  visual=(16, 1100)), 100, {}),
     # the largest window block the kernels take: G W = 512 rows at d = 128
     ("rows_512_d128", dict(seq_len=1500, layers=2, q_heads=16, kv_heads=2, head_dim=128,
                            window=64, visual=(16, 1400)), 200, {}),
