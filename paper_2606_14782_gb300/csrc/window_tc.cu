@@ -88,14 +88,15 @@ __host__ __device__ inline Smem smem_layout(const Plan& p)
     // two tiles
     s.bars = s.xchg + (PASS == 1 ? 4u : 2u) * kGroups * 128u * 8u;
     s.bars = (s.bars + 7u) & ~7u;
-    s.total = s.bars + 144u + 8u * (2u * (uint32_t)p.stages + 16u);  // barriers, TMEM base, abort flag
+    s.total = s.bars + 272u + 16u * (uint32_t)p.stages;  // barriers, TMEM base, abort flag
     return s;
 }
 
 // Barrier block, 8-byte slots from `base` (a shared-memory address):
 // t_full[4], t_empty[4], q_full, q_empty, drain, five spare slots, the
-// TMEM base word, the abort word, then k_full[stages], k_empty[stages],
-// x_full[2][4], x_empty[2][4].
+// TMEM base word, the abort word, x_full[2][4], x_empty[2][4] (fixed
+// offsets, so the epilogue's barrier addresses need no stage count), then
+// k_full[stages], k_empty[stages].
 struct Bars {
     uint32_t base;
     int stages;
@@ -106,20 +107,17 @@ struct Bars {
     __device__ __forceinline__ uint32_t drain() const { return base + 80u; }
     __device__ __forceinline__ uint32_t tmem_slot() const { return base + 128u; }
     __device__ __forceinline__ uint32_t abort() const { return base + 136u; }
-    __device__ __forceinline__ uint32_t k_full(int st) const { return base + 144u + 8u * st; }
-    __device__ __forceinline__ uint32_t k_empty(int st) const
-    {
-        return base + 144u + 8u * (stages + st);
-    }
-    // pass 2, exchange slot p (tile parity) of lane quarter q: the three
-    // non-merging groups' partial sums are in it / the merging group has read it
-    __device__ __forceinline__ uint32_t x_full(int p, int q) const
-    {
-        return base + 144u + 8u * (2 * stages + 4 * p + q);
-    }
+    // exchange slot p of lane quarter q (pass 1: p = 0 only): the three
+    // non-merging groups' partials are in it / the merging group has read it
+    __device__ __forceinline__ uint32_t x_full(int p, int q) const { return base + 144u + 8u * (4 * p + q); }
     __device__ __forceinline__ uint32_t x_empty(int p, int q) const
     {
-        return base + 144u + 8u * (2 * stages + 8 + 4 * p + q);
+        return base + 208u + 8u * (4 * p + q);
+    }
+    __device__ __forceinline__ uint32_t k_full(int st) const { return base + 272u + 8u * st; }
+    __device__ __forceinline__ uint32_t k_empty(int st) const
+    {
+        return base + 272u + 8u * (stages + st);
     }
 };
 
