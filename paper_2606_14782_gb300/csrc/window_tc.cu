@@ -421,15 +421,20 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
         // partial: group n mod 4 of this CTA's n-th chunk waits until the
         // other three groups of its lane quarter have left their (max, sum)
         // per row block in shared memory, merges them in group order and
-        // frees the slot for the next chunk
+        // frees the slot for the next chunk.  Every group, the merging one
+        // included, first waits for the slot's previous read: a parity wait
+        // is unambiguous only once the barrier's previous phase has
+        // completed, and the merging group's x_full wait could otherwise pass
+        // on the previous chunk's phase while a slower group is a chunk
+        // behind.
         const int merger = nch & 3;
         const uint32_t ph = (uint32_t)nch & 1u;
         ++nch;
+        if (!tc::mbar_wait(b.x_empty(0, quarter), ph ^ 1u, b.abort())) {
+            ok = false;
+            break;
+        }
         if (group != merger) {
-            if (!tc::mbar_wait(b.x_empty(0, quarter), ph ^ 1u, b.abort())) {
-                ok = false;
-                break;
-            }
 #pragma unroll
             for (int rb = 0; rb < 4; ++rb) {
                 if (rb >= nrb) break;
@@ -638,17 +643,21 @@ __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, 
             // slots, used by this CTA's tiles in turn); group n mod 4 of the
             // CTA's n-th tile adds them in group order once the other three
             // have arrived on the slot's barrier, frees the slot and stores
-            // the token's B, Q and E
+            // the token's B, Q and E.  Every group, the merging one included,
+            // first waits for the slot's previous read, so that the merging
+            // group's parity wait on x_full cannot pass on the slot's previous
+            // phase (with four TMEM buffers a group can run two tiles ahead
+            // of another).
             const int par = ntile & 1;
             const uint32_t ph = (uint32_t)(ntile >> 1) & 1u;
             const int merger = ntile & 3;
             ++ntile;
             float2* slot = xs + (size_t)(par * kGroups) * 128 + quarter * 32 + lane;
+            if (!tc::mbar_wait(b.x_empty(par, quarter), ph ^ 1u, b.abort())) {
+                ok = false;
+                break;
+            }
             if (group != merger) {
-                if (!tc::mbar_wait(b.x_empty(par, quarter), ph ^ 1u, b.abort())) {
-                    ok = false;
-                    break;
-                }
                 slot[group * 128] = make_float2(bsum, qsum);
                 __syncwarp();
                 if (lane == 0) tc::mbar_arrive(b.x_full(par, quarter));
