@@ -48,6 +48,8 @@ struct Smem {
     // offsets in bytes from the 1024-aligned dynamic shared memory base
     uint32_t q, k, ones, bias, xchg, bars;
     uint32_t q_half;      // bytes of one 64-column half of the window rows
+    uint32_t q_slot;      // bytes of one slot of window rows (both halves)
+    uint32_t bias_slot;   // bytes of one slot of the pass-2 bias operand
     uint32_t k_stage;     // bytes of one K tile
     uint32_t total;
 };
@@ -67,6 +69,7 @@ struct Smem {
 // so every group of 8 token rows reads the same atom.
 struct Plan {
     int q_rows, n_jobs, granules, stages, nbuf_log2, bias_rows, ones_atom;
+    int q_slots;  // 2: the next unit's window rows load while this unit's MMAs run
 };
 
 constexpr uint32_t kOnesBytes = 128u * 128u;
@@ -78,12 +81,14 @@ __host__ __device__ inline Smem smem_layout(const Plan& p)
     Smem s;
     constexpr int H = D / 64;
     s.q_half = (uint32_t)p.q_rows * 128u;
+    s.q_slot = H * s.q_half;
+    s.bias_slot = PASS == 2 ? (uint32_t)p.bias_rows * 128u : 0u;
     s.k_stage = (uint32_t)H * kTileTok * 128u;
     s.q = 0;
-    s.k = s.q + H * s.q_half;
+    s.k = s.q + (uint32_t)p.q_slots * s.q_slot;
     s.ones = s.k + (uint32_t)p.stages * s.k_stage;
     s.bias = s.ones + (PASS == 2 ? (p.ones_atom ? kOnesAtomBytes : kOnesBytes) : 0u);
-    s.xchg = s.bias + (PASS == 2 ? (uint32_t)p.bias_rows * 128u : 0u);
+    s.xchg = s.bias + (uint32_t)p.q_slots * s.bias_slot;
     // every group's partials: pass 1 per row block of a chunk, pass 2 for
     // two tiles
     s.bars = s.xchg + (PASS == 1 ? 4u : 2u) * kGroups * 128u * 8u;
@@ -93,7 +98,8 @@ __host__ __device__ inline Smem smem_layout(const Plan& p)
 }
 
 // Barrier block, 8-byte slots from `base` (a shared-memory address):
-// t_full[4], t_empty[4], q_full, q_empty, drain, five spare slots, the
+// t_full[4], t_empty[4], q_full[0], q_empty[0], drain, q_full[1],
+// q_empty[1], three spare slots, the
 // TMEM base word, the abort word, x_full[2][4], x_empty[2][4] (fixed
 // offsets, so the epilogue's barrier addresses need no stage count), then
 // k_full[stages], k_empty[stages].
@@ -102,8 +108,8 @@ struct Bars {
     int stages;
     __device__ __forceinline__ uint32_t t_full(int i) const { return base + 8u * i; }
     __device__ __forceinline__ uint32_t t_empty(int i) const { return base + 32u + 8u * i; }
-    __device__ __forceinline__ uint32_t q_full() const { return base + 64u; }
-    __device__ __forceinline__ uint32_t q_empty() const { return base + 72u; }
+    __device__ __forceinline__ uint32_t q_full(int slot) const { return base + (slot ? 88u : 64u); }
+    __device__ __forceinline__ uint32_t q_empty(int slot) const { return base + (slot ? 96u : 72u); }
     __device__ __forceinline__ uint32_t drain() const { return base + 80u; }
     __device__ __forceinline__ uint32_t tmem_slot() const { return base + 128u; }
     __device__ __forceinline__ uint32_t abort() const { return base + 136u; }
@@ -206,7 +212,7 @@ __device__ __forceinline__ void write_bias(const TcArgs& a, uint8_t* bias, int u
 // (pass 2 also rewrites the bias operand, a second arrival on q_full).
 template <int D, int PASS>
 __device__ __forceinline__ void produce(const TcArgs& a, const Smem& L, uint8_t* sm, const Bars& b,
-                                        int stages, int q_rows, const JobTable& jt)
+                                        int stages, int q_rows, int q_slots, const JobTable& jt)
 {
     constexpr int H = D / 64;
     const Shape& s = a.s;
@@ -221,20 +227,22 @@ __device__ __forceinline__ void produce(const TcArgs& a, const Smem& L, uint8_t*
         const int u = g / a.chunks, ci = g - u * a.chunks;
         const int pair = u / s.hkv, h = u - pair * s.hkv;
         if (u != cur_u) {
-            ok = __all_sync(0xffffffffu, tc::mbar_wait(b.q_empty(), (qloads & 1) ^ 1, b.abort()));
+            const int slot = qloads % q_slots, use = qloads / q_slots;
+            ok = __all_sync(0xffffffffu, tc::mbar_wait(b.q_empty(slot), (use & 1) ^ 1, b.abort()));
             if (!ok) break;
+            uint8_t* qdst = sm + L.q + slot * L.q_slot;
             if (lane == 0) {
-                tc::mbar_arrive_expect_tx(b.q_full(), H * L.q_half);
+                tc::mbar_arrive_expect_tx(b.q_full(slot), L.q_slot);
                 for (int kh = 0; kh < H; ++kh)
                     for (int rb = 0; rb < q_rows / kQBox; ++rb)
-                        tc::tma_load_2d(sm + L.q + kh * L.q_half + rb * kQBox * 128, a.qmaps + pair,
-                                        kh * 64, h * s.rows + rb * kQBox, b.q_full());
+                        tc::tma_load_2d(qdst + kh * L.q_half + rb * kQBox * 128, a.qmaps + pair,
+                                        kh * 64, h * s.rows + rb * kQBox, b.q_full(slot));
             }
             if (PASS == 2) {
-                write_bias(a, sm + L.bias, u, jt, inv_c);
+                write_bias(a, sm + L.bias + slot * L.bias_slot, u, jt, inv_c);
                 tc::fence_proxy_async_smem();
                 __syncwarp();
-                if (lane == 0) tc::mbar_arrive(b.q_full());
+                if (lane == 0) tc::mbar_arrive(b.q_full(slot));
             }
             ++qloads;
             cur_u = u;
@@ -260,7 +268,10 @@ __device__ __forceinline__ void produce(const TcArgs& a, const Smem& L, uint8_t*
         const int last = kt - 1 - ((kt - 1 - st) % stages);
         tc::mbar_wait(b.k_full(st), (last / stages) & 1, 0u);
     }
-    if (qloads > 0) tc::mbar_wait(b.q_full(), (qloads - 1) & 1, 0u);
+    for (int slot = 0; slot < q_slots && slot < qloads; ++slot) {
+        const int last = qloads - 1 - ((qloads - 1 - slot) % q_slots);
+        tc::mbar_wait(b.q_full(slot), (last / q_slots) & 1, 0u);
+    }
 }
 
 // ------------------------------------------------------ MMA issuer (warp 1)
@@ -269,7 +280,7 @@ __device__ __forceinline__ void produce(const TcArgs& a, const Smem& L, uint8_t*
 // Pass 2: A = K tile (M = 128 tokens), B = window rows (N = n_h per half).
 template <int D, int PASS, int NBUF_LOG2>
 __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* sm, const Bars& b, int stages,
-                      const JobTable& jt, uint32_t ones_stride)
+                      int q_slots, const JobTable& jt, uint32_t ones_stride)
 {
     const Shape& s = a.s;
     const int ntiles = (s.N + kTileTok - 1) / kTileTok;
@@ -279,16 +290,18 @@ __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* s
     constexpr uint32_t buf_cols = (uint32_t)kTmemCols >> NBUF_LOG2;
     int c0, c1;
     chunk_range(a.total_chunks, &c0, &c1);
-    int cur_u = -1, qwaits = 0, kt = 0, job = 0;
+    int cur_u = -1, cur_slot = 0, qwaits = 0, kt = 0, job = 0;
     bool ok = true;
     for (int g = c0; g < c1 && ok; ++g) {
         const int u = g / a.chunks, ci = g - u * a.chunks;
         if (u != cur_u) {
-            if (cur_u >= 0) tc::umma_commit(b.q_empty());  // previous unit's MMAs release Q
-            if (!tc::mbar_wait(b.q_full(), qwaits & 1, b.abort())) { ok = false; break; }
+            if (cur_u >= 0) tc::umma_commit(b.q_empty(cur_slot));  // previous unit's MMAs release its slot
+            const int slot = qwaits % q_slots, use = qwaits / q_slots;
+            if (!tc::mbar_wait(b.q_full(slot), use & 1, b.abort())) { ok = false; break; }
             tc::fence_after_sync();
             ++qwaits;
             cur_u = u;
+            cur_slot = slot;
         }
         const int t1 = min(ntiles, (ci + 1) * kTilesPerChunk);
         for (int t = ci * kTilesPerChunk; t < t1 && ok; ++t, ++kt) {
@@ -305,10 +318,10 @@ __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* s
                 tc::fence_after_sync();
                 const uint32_t d_tmem = tmem + buf * buf_cols;
                 const uint32_t idesc = tc::idesc_bf16(128, jt.n(j));
-                const uint32_t qaddr = sbase + L.q + jt.row0(j) * 128;
+                const uint32_t qaddr = sbase + L.q + cur_slot * L.q_slot + jt.row0(j) * 128;
                 if (PASS == 2)  // D = -lse2 / c per row (columns of D), then += K Q^T
                     tc::umma_bf16(d_tmem, tc::sdesc_sw128(sbase + L.ones, ones_stride),
-                                  tc::sdesc_sw128(sbase + L.bias + 32 * j), idesc, 0);
+                                  tc::sdesc_sw128(sbase + L.bias + cur_slot * L.bias_slot + 32 * j), idesc, 0);
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
                     const int kh = kk / 4;
@@ -744,8 +757,10 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, Plan p
             tc::mbar_init(b.t_full(i), 1);
             tc::mbar_init(b.t_empty(i), kEpiThreads / 32);  // one arrival per epilogue warp
         }
-        tc::mbar_init(b.q_full(), PASS == 2 ? 2 : 1);  // pass 2: TMA bytes + the bias writes
-        tc::mbar_init(b.q_empty(), 1);
+        for (int slot = 0; slot < 2; ++slot) {
+            tc::mbar_init(b.q_full(slot), PASS == 2 ? 2 : 1);  // pass 2: TMA bytes + the bias writes
+            tc::mbar_init(b.q_empty(slot), 1);
+        }
         tc::mbar_init(b.drain(), 1);
         for (int i = 0; i < 8; ++i) {
             tc::mbar_init(b.x_full(i >> 2, i & 3), kGroups - 1);
@@ -763,7 +778,7 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, Plan p
         // 8 rows when ones_atom); the bias operand starts zeroed (the
         // producer fills columns 16 j .. 16 j + 2)
         const int row = threadIdx.x - 64;
-        for (int rr = row; rr < pl.bias_rows; rr += 128) {
+        for (int rr = row; rr < pl.q_slots * pl.bias_rows; rr += 128) {
             uint4* bias = reinterpret_cast<uint4*>(sm + L.bias + rr * 128);
             for (int q = 0; q < 8; ++q) bias[q] = make_uint4(0u, 0u, 0u, 0u);
         }
@@ -781,14 +796,14 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, Plan p
     tc::fence_after_sync();
 
     if (warp == 0) {
-        produce<D, PASS>(a, L, sm, b, pl.stages, pl.q_rows, jt);
+        produce<D, PASS>(a, L, sm, b, pl.stages, pl.q_rows, pl.q_slots, jt);
     } else if (warp == 1) {
         if (tc::elect_one()) {
             const uint32_t ones_stride = pl.ones_atom ? 0u : 1024u;
             if (pl.nbuf_log2 == 1)
-                issue<D, PASS, 1>(a, L, sm, b, pl.stages, jt, ones_stride);
+                issue<D, PASS, 1>(a, L, sm, b, pl.stages, pl.q_slots, jt, ones_stride);
             else
-                issue<D, PASS, 2>(a, L, sm, b, pl.stages, jt, ones_stride);
+                issue<D, PASS, 2>(a, L, sm, b, pl.stages, pl.q_slots, jt, ones_stride);
         }
     } else {
         if (PASS == 1)
@@ -847,11 +862,16 @@ cudaError_t launch_impl(const TcArgs& a, cudaStream_t st)
         pl.granules = PASS == 1 ? 8 * pl.n_jobs : granules;
         pl.nbuf_log2 = per_job == 16 ? 1 : 2;
         pl.bias_rows = PASS == 2 ? 16 * ((pl.granules + pl.n_jobs - 1) / pl.n_jobs) : 0;
+        // two slots of window rows when they fit beside at least three K
+        // stages, else one
         for (pl.ones_atom = 0; pl.ones_atom < 2 && !fits; ++pl.ones_atom) {
-            for (pl.stages = 4; pl.stages > 2; --pl.stages)
-                if (smem_layout<D, PASS>(pl).total <= budget) break;
-            L = smem_layout<D, PASS>(pl);
-            fits = L.total <= budget;
+            for (int qs = 2; qs >= 1 && !fits; --qs) {
+                pl.q_slots = qs;
+                for (pl.stages = 4; pl.stages > 2; --pl.stages)
+                    if (smem_layout<D, PASS>(pl).total <= budget) break;
+                L = smem_layout<D, PASS>(pl);
+                fits = L.total <= budget && (qs == 1 || pl.stages >= 3);
+            }
             if (fits) break;
         }
     }
