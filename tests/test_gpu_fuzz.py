@@ -9,14 +9,19 @@ once from a fixed seed: window sizes from 1 to 64 (multiples of 16 and
 not), query-head groups of 1 to 8, head dim 64 and 128, prompt lengths that
 end mid-tile and mid-chunk, budgets from the window alone to more than the
 prompt, and calls with more chunks than the GPU has SMs (so that CTA ranges
-cross unit boundaries after short or odd-length units).
+cross unit boundaries after short or odd-length units).  The same shapes go
+through the layer-by-layer path (one layer per call, bit-identical to the
+whole step) and the path that takes the prefill's row normalisers (one
+window pass; within the parity tolerance of the whole step).
 """
 
 import numpy as np
 import pytest
+import torch
 
 from paper_2606_14782_gb300 import bacon, build, workloads
-from test_gpu_parity import compare, oracle_run, run_gpu
+from parity import check_scores
+from test_gpu_parity import compare, oracle_run, prefill_lse, run_gpu
 
 pytestmark = pytest.mark.gpu
 
@@ -72,3 +77,41 @@ def test_random_shapes(name, over, budget):
     # each window softmax row sums to one, so B and Q do per unit
     np.testing.assert_allclose(gpu["B"].sum(-1), 1.0, atol=2e-4)
     np.testing.assert_allclose(gpu["Q"].sum(-1), 1.0, atol=2e-4)
+
+
+@pytest.mark.parametrize("name,over,budget", SHAPES, ids=[s[0] for s in SHAPES])
+def test_random_shapes_layer_path(name, over, budget):
+    wl = workloads.CONFIGS["tiny"].with_(**over)
+    x = workloads.generate(wl, seed=11, device="cuda")
+    whole = run_gpu(wl, x, budget)
+    p = bacon.default_params(max_seq_len=wl.seq_len, max_requests=wl.requests)
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool,
+                        budget, params=p)
+    st = bacon.State(ctx)
+    r = wl.requests - 1
+    for l in range(wl.layers):
+        S = st.score_layer(l, x.qwin[r, l], x.k[r, l], scores_out=True)
+        idx = st.select(budget, wl.seq_len)
+        ko, vo = ctx.compact(x.k[r, l], x.v[r, l], idx)
+        ctx.sync()
+        assert np.array_equal(S.cpu().numpy(), whole["S"][r, l]), l
+        assert np.array_equal(idx.cpu().numpy(), whole["idx"][r, l]), l
+        assert torch.equal(ko.cpu(), whole["Kc"][r, l]) and torch.equal(vo.cpu(), whole["Vc"][r, l])
+    st.close()
+    ctx.close()
+
+
+@pytest.mark.parametrize("name,over,budget", SHAPES, ids=[s[0] for s in SHAPES])
+def test_random_shapes_prefill_normalisers(name, over, budget):
+    wl = workloads.CONFIGS["tiny"].with_(**over)
+    x = workloads.generate(wl, seed=11, device="cuda")
+    whole = run_gpu(wl, x, budget)
+    p = bacon.default_params(keep_scores=1, max_seq_len=wl.seq_len, max_requests=wl.requests)
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool,
+                        budget, params=p)
+    ctx.compress_with_lse(x.qwin, x.k, x.v, prefill_lse(wl, x), budget)
+    ctx.sync()
+    shp = (wl.requests, wl.layers, wl.kv_heads, wl.seq_len)
+    for kind in ("B", "Q", "E"):
+        check_scores(f"{name} {kind}", ctx.scores(kind).cpu().numpy().reshape(shp), whole[kind])
+    ctx.close()
