@@ -1,0 +1,214 @@
+"""Model of the window kernels' synchronisation, run on the CPU.
+
+One CTA of a window pass has a producer (TMA loads of K tiles into a ring of
+stages and of the window rows into one or two slots), an MMA thread (waits
+for the operands and for free TMEM buffers, commits its MMAs to mbarriers)
+and sixteen epilogue warps (wait for accumulators, free the buffers, and hand
+partial results to a rotating merging group through shared-memory slots
+guarded by x_full / x_empty barriers).  mbarrier waits test a phase parity,
+so each wait is correct only while the barrier is exactly one phase past the
+one the waiter expects when the wait returns.  The model replays the
+kernels' sequence of waits and arrivals (TMA completions and MMA commits
+arrive asynchronously, commits in issue order) under random interleavings,
+on work lists cut the way the kernels cut them (each CTA a contiguous range
+of 1024-token chunks over (request, layer, kv-head) units), and checks that
+every schedule finishes and every wait returns in its own phase.  The
+variant in which the merging group does not first wait for the slot's
+previous read (the kernels' earlier protocol) fails the check.
+"""
+
+import random
+
+import pytest
+
+
+class Bar:
+    """An mbarrier: `count` arrivals complete a phase."""
+
+    def __init__(self, count, name):
+        self.count, self.pending, self.phase, self.name = count, count, 0, name
+
+    def arrive(self):
+        self.pending -= 1
+        assert self.pending >= 0, self.name
+        if self.pending == 0:
+            self.phase += 1
+            self.pending = self.count
+
+
+class Fault(Exception):
+    pass
+
+
+def wait(bar, k):
+    """Generator: wait for completion of phase k with a parity test; checks the
+    barrier is exactly one phase past k when the wait returns."""
+    while (bar.phase & 1) == (k & 1):
+        yield
+    if bar.phase != k + 1:
+        raise Fault(f"{bar.name}: waited for phase {k}, barrier at phase {bar.phase}")
+
+
+def simulate(chunks, n_tiles, tpc, jobs_per_tile, nbuf, stages, q_slots, pass2, guard, seed):
+    """chunks: the CTA's list of (unit, chunk index); n_tiles: tiles per unit."""
+    rnd = random.Random(seed)
+    t_full = [Bar(1, f"t_full{i}") for i in range(nbuf)]
+    t_empty = [Bar(16, f"t_empty{i}") for i in range(nbuf)]
+    k_full = [Bar(1, f"k_full{i}") for i in range(stages)]
+    k_empty = [Bar(1, f"k_empty{i}") for i in range(stages)]
+    q_full = [Bar(2 if pass2 else 1, f"q_full{i}") for i in range(q_slots)]
+    q_empty = [Bar(1, f"q_empty{i}") for i in range(q_slots)]
+    x_full = {(p, q): Bar(3, f"x_full{p}{q}") for p in range(2) for q in range(4)}
+    x_empty = {(p, q): Bar(1, f"x_empty{p}{q}") for p in range(2) for q in range(4)}
+    drain = Bar(1, "drain")
+    tma = []       # pending TMA completions (any order)
+    commits = []   # pending MMA-commit arrivals (in issue order)
+
+    def tiles_of(ci):
+        return range(ci * tpc, min(n_tiles, (ci + 1) * tpc))
+
+    def producer():
+        cur, qloads, kt = -1, 0, 0
+        for u, ci in chunks:
+            if u != cur:
+                slot, use = qloads % q_slots, qloads // q_slots
+                yield from wait(q_empty[slot], use - 1)
+                tma.append(q_full[slot])
+                if pass2:
+                    yield
+                    q_full[slot].arrive()
+                qloads += 1
+                cur = u
+            for _ in tiles_of(ci):
+                st, n = kt % stages, kt // stages
+                yield from wait(k_empty[st], n - 1)
+                tma.append(k_full[st])
+                kt += 1
+                yield
+        for st in range(min(stages, kt)):
+            last = kt - 1 - ((kt - 1 - st) % stages)
+            yield from wait(k_full[st], last // stages)
+        for slot in range(min(q_slots, qloads)):
+            last = qloads - 1 - ((qloads - 1 - slot) % q_slots)
+            yield from wait(q_full[slot], last // q_slots)
+
+    def mma():
+        cur, cur_slot, qwaits, kt, job = -1, 0, 0, 0, 0
+        for u, ci in chunks:
+            if u != cur:
+                if cur >= 0:
+                    commits.append(q_empty[cur_slot])
+                slot, use = qwaits % q_slots, qwaits // q_slots
+                yield from wait(q_full[slot], use)
+                qwaits += 1
+                cur, cur_slot = u, slot
+            for _ in tiles_of(ci):
+                st, n = kt % stages, kt // stages
+                yield from wait(k_full[st], n)
+                kt += 1
+                for _ in range(jobs_per_tile):
+                    buf, nb = job % nbuf, job // nbuf
+                    job += 1
+                    yield from wait(t_empty[buf], nb - 1)
+                    commits.append(t_full[buf])
+                    yield
+                commits.append(k_empty[st])
+        commits.append(drain)
+        yield from wait(drain, 0)
+
+    def epilogue(q, g):
+        job = n = 0
+        for u, ci in chunks:
+            ts = list(tiles_of(ci))
+            for i, _ in enumerate(ts):
+                for _ in range(jobs_per_tile):
+                    buf, nb = job % nbuf, job // nbuf
+                    job += 1
+                    yield from wait(t_full[buf], nb)
+                    yield
+                    t_empty[buf].arrive()
+                last_of_chunk = i == len(ts) - 1
+                if not pass2 and not last_of_chunk:
+                    continue
+                slots = 2 if pass2 else 1
+                par, use, merger = n % slots, n // slots, n & 3
+                n += 1
+                if g != merger or guard:
+                    yield from wait(x_empty[(par, q)], use - 1)
+                if g != merger:
+                    yield
+                    x_full[(par, q)].arrive()
+                else:
+                    yield from wait(x_full[(par, q)], use)
+                    yield
+                    x_empty[(par, q)].arrive()
+
+    procs = [producer(), mma()] + [epilogue(q, g) for q in range(4) for g in range(4)]
+    live = list(range(len(procs)))
+    for _ in range(500000):
+        if not live and not tma and not commits:
+            return None
+        r = rnd.random()
+        if tma and r < 0.25:
+            tma.pop(rnd.randrange(len(tma))).arrive()
+            continue
+        if commits and r < 0.5:
+            commits.pop(0).arrive()
+            continue
+        if not live:
+            continue
+        i = rnd.choice(live)
+        try:
+            next(procs[i])
+        except StopIteration:
+            live.remove(i)
+        except Fault as f:
+            return str(f)
+    return "deadlock"
+
+def cta_range(units, chunks_per_unit, total_ctas, cta):
+    total = units * chunks_per_unit
+    c0, c1 = cta * total // total_ctas, (cta + 1) * total // total_ctas
+    return [(g // chunks_per_unit, g % chunks_per_unit) for g in range(c0, c1)]
+
+
+def cta_range(units, chunks_per_unit, total_ctas, cta):
+    total = units * chunks_per_unit
+    c0, c1 = cta * total // total_ctas, (cta + 1) * total // total_ctas
+    return [(g // chunks_per_unit, g % chunks_per_unit) for g in range(c0, c1)]
+
+
+def _cases(n=40, seed=3):
+    rng = random.Random(seed)
+    out = []
+    while len(out) < n:
+        n_tiles = rng.choice([1, 3, 8, 9, 11, 16, 51, 128])
+        cpu = -(-n_tiles // 8)
+        units = rng.randint(1, 12)
+        ctas = rng.randint(1, max(1, units * cpu))
+        chunks = cta_range(units, cpu, ctas, rng.randrange(ctas))
+        if not chunks or len(chunks) > 24:
+            continue
+        pass2 = rng.random() < 0.5
+        if pass2:
+            jobs, nbuf = rng.choice([(1, 4), (2, 2), (2, 4), (1, 2)])
+        else:
+            jobs, nbuf = rng.choice([1, 2, 3, 4]), 4
+        out.append((chunks, n_tiles, jobs, nbuf, rng.choice([2, 3, 4]), rng.choice([1, 2]), pass2))
+    return out
+
+
+@pytest.mark.parametrize("chunks,n_tiles,jobs,nbuf,stages,q_slots,pass2", _cases())
+def test_pipeline_finishes_and_waits_in_phase(chunks, n_tiles, jobs, nbuf, stages, q_slots, pass2):
+    for seed in range(6):
+        fault = simulate(chunks, n_tiles, 8, jobs, nbuf, stages, q_slots, pass2, True, seed)
+        assert fault is None, (seed, fault)
+
+
+def test_model_catches_the_unguarded_merger():
+    # one job per tile and four TMEM buffers let an epilogue group run two
+    # tiles ahead of another; without the extra wait the merging group's
+    # x_full wait passes on the slot's previous phase
+    chunks = cta_range(3, 2, 1, 0)
+    faults = [simulate(chunks, 11, 8, 1, 4, 4, 1, True, False, s) for s in range(8)]
+    assert any(f is not None for f in faults)
