@@ -315,7 +315,7 @@ def main():
     }
     total = sum(t for t, _ in prof.values())
     kernels = {k: {"ms_per_launch": (t / n if n else None), "share": (t / total if total else None)}
-               for k, (t, n) in prof.items()}
+               for k, (t, n) in prof.items() if n}
     dom = max(prof, key=lambda k: prof[k][0])
     dom_ms = prof[dom][0] / max(1, prof[dom][1])
     achieved_gbs = algo_bytes[dom] / (dom_ms / 1e3) / 1e9
@@ -344,7 +344,7 @@ def main():
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded, paper-shaped; no datasets)",
             "config": config_dict(wl, budget, world),
-            "gpu_launches": 5 * args.steps, "roofline": roofline, "kernels": kernels,
+            "gpu_launches": sum(n for _, n in prof.values()), "roofline": roofline, "kernels": kernels,
             "clocks": clocks}
 
     if not args.no_extras:

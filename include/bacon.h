@@ -287,7 +287,11 @@ bacon_status bacon_profile_enable(bacon_ctx* ctx, int enable);
 
 /* Waits for the recorded work, then writes per stage the summed device time
  * in ms and the launch count since the previous read (arrays of at least
- * `n` entries; n <= BACON_PROFILE_STAGES), and clears the record. */
+ * `n` entries; n <= BACON_PROFILE_STAGES), and clears the record.  A stage
+ * that launched nothing in a call is not counted: when every unit's logits
+ * fit in tensor memory (at most 32 window rows and 1024 tokens) the window
+ * score is one kernel, reported as window_scores, with no window_stats or
+ * window_combine launch. */
 bacon_status bacon_profile_read(bacon_ctx* ctx, double* ms, int* launches, int n);
 
 /* Window scores of one layer (B, Q and E of Eqs. 1, 2 and 4 for every

@@ -112,6 +112,7 @@ struct bacon_ctx {
     int prof_on = 0;
     std::vector<cudaEvent_t> ev_free;
     std::vector<std::vector<cudaEvent_t>> ev_pending;  // 6 events per call
+    std::vector<uint32_t> ev_skipped;                  // per call: stages that launched nothing
 };
 
 struct bacon_state {
@@ -248,6 +249,7 @@ void free_ctx_buffers(bacon_ctx* c)
     for (cudaEvent_t e : c->ev_free)
         if (e) cudaEventDestroy(e);
     c->ev_pending.clear();
+    c->ev_skipped.clear();
     c->ev_free.clear();
     void* bufs[] = {c->B,      c->Q,      c->E,      c->S,      c->V,      c->Bp,
                     c->lam,    c->lse2,   c->partial, c->err,   c->hq_buf, c->hk_buf,
@@ -275,13 +277,18 @@ struct StageEvents {
             ev.push_back(e);
         }
     }
+    uint32_t skipped = 0;
     void mark(int i)
     {
         if (c->prof_on && ev[i]) cudaEventRecord(ev[i], st);
     }
+    void skip(int i) { skipped |= 1u << i; }  // stage i launched nothing in this call
     void commit()
     {
-        if (c->prof_on) c->ev_pending.push_back(ev);
+        if (c->prof_on) {
+            c->ev_pending.push_back(ev);
+            c->ev_skipped.push_back(skipped);
+        }
         ev.clear();
     }
     ~StageEvents()
@@ -308,8 +315,20 @@ bacon_status window_passes(bacon_ctx* c, const Shape& s, const void* const* q,
     const TcArgs ta = tc_args(s, c->d_maps, c->d_maps + kMaxPairs, partial, lse2,
                               c->B + unit0 * N, c->Q + unit0 * N, c->E + unit0 * N, c->err);
     prof.mark(0);
+    if (!prefill_lse && window_onepass_fits(s)) {
+        // the unit's logits stay in tensor memory: one kernel, one pass over K
+        // (timed as the scores stage)
+        prof.mark(1);
+        prof.mark(2);
+        prof.skip(0);
+        prof.skip(1);
+        BACON_CUDA(launch_window_onepass(ta, st), "window_onepass launch");
+        prof.mark(3);
+        return BACON_OK;
+    }
     if (prefill_lse) {
         prof.mark(1);
+        prof.skip(0);
         LseTable t;
         for (int i = 0; i < pairs; ++i) t.lse[i] = prefill_lse[i];
         BACON_CUDA(launch_lse_from_prefill(s, t, lse2, st), "normaliser conversion launch");
@@ -1082,10 +1101,13 @@ bacon_status bacon_profile_read(bacon_ctx* ctx, double* ms, int* launches, int n
         launches[i] = 0;
     }
     bacon_status rc = BACON_OK;
-    for (auto& v : ctx->ev_pending) {
+    for (size_t c = 0; c < ctx->ev_pending.size(); ++c) {
+        auto& v = ctx->ev_pending[c];
+        const uint32_t skipped = c < ctx->ev_skipped.size() ? ctx->ev_skipped[c] : 0u;
         if (v.back() && cudaEventSynchronize(v.back()) != cudaSuccess) rc = fail(BACON_ECUDA, "event wait failed");
         for (int i = 0; i < n && rc == BACON_OK; ++i) {
             float t = 0.f;
+            if ((skipped >> i) & 1u) continue;
             if (v[i] && v[i + 1] && cudaEventElapsedTime(&t, v[i], v[i + 1]) == cudaSuccess) {
                 ms[i] += t;
                 launches[i] += 1;
@@ -1095,6 +1117,7 @@ bacon_status bacon_profile_read(bacon_ctx* ctx, double* ms, int* launches, int n
             if (e) ctx->ev_free.push_back(e);
     }
     ctx->ev_pending.clear();
+    ctx->ev_skipped.clear();
     return rc;
 }
 

@@ -1,0 +1,411 @@
+// Window scores (Eqs. 1, 2, 4) in one pass over K, for units whose logits fit
+// in tensor memory: at most 32 window rows (G W <= 32) and at most 1024
+// tokens, i.e. 8 tiles x 32 columns, so that two units' logits (2 x 256 of
+// the 512 TMEM columns) are resident at once.
+//
+// The two-pass kernels (window_tc.cu) stream K twice because a softmax row
+// must be normalised over all N keys before any token's share is final.
+// When a whole unit's logits stay in TMEM, the normaliser is computed from
+// them and the same logits are read again for the shares, so K is read once:
+//   * warp 0 loads the unit's window rows (one of two slots) and its K tiles
+//     (a ring of stages) by TMA;
+//   * warp 1 computes D[token][row] = K Q^T (M = 128 tokens per tile, N = 32
+//     rows) for every tile of the unit into the unit's half of TMEM and
+//     commits it;
+//   * eight epilogue warps (two groups x four lane quarters; group g takes
+//     the tiles t = g mod 2) reduce each row's maximum over their tokens by a
+//     butterfly transpose across the warp's lanes, meet at a CTA-wide
+//     mbarrier, reduce the sums of 2^(x - max) the same way, meet again, and
+//     then each thread sums its token's shares over the rows (B), over the
+//     last-position rows (Q) and stores E = [Q - B]_+.
+// Every wait is bounded (abort flag, clock limit): on timeout the CTA records
+// BACON_ETIMEOUT, drains its own copies and MMAs, frees TMEM and returns.
+#include <cuda_bf16.h>
+
+#include "tc.cuh"
+#include "window_tc.h"
+
+namespace bacon {
+namespace {
+
+constexpr int kTok = 128;        // tokens per K tile (TMEM lanes)
+constexpr int kRows = 32;        // window rows per unit, padded (MMA N)
+constexpr int kMaxTiles = 8;     // tiles per unit
+constexpr int kSlotCols = 256;   // TMEM columns of one unit
+constexpr int kEpiWarps = 8;      // two groups of four lane quarters
+constexpr int kGroups = kEpiWarps / 4;
+constexpr int kThreads = 64 + 32 * kEpiWarps;
+constexpr int kStages = 4;
+constexpr float kLog2e = 1.4426950408889634f;
+
+struct Layout {
+    uint32_t q_half, q_slot, k_stage;  // bytes
+    uint32_t q, k, xr, xs, fm, bars, total;
+};
+
+template <int D>
+__host__ __device__ inline Layout layout()
+{
+    constexpr int H = D / 64;
+    Layout L;
+    L.q_half = (uint32_t)kTcQBoxRows * 128u;  // one 64-row box (rows beyond 32 unused)
+    L.q_slot = H * L.q_half;
+    L.k_stage = (uint32_t)H * kTok * 128u;
+    L.q = 0;
+    L.k = L.q + 2 * L.q_slot;
+    L.xr = L.k + kStages * L.k_stage;             // [warp][row] partial maxima
+    L.xs = L.xr + kEpiWarps * kRows * 4u;          // [warp][row] partial sums
+    L.fm = L.xs + kEpiWarps * kRows * 4u;          // [warp][row] the rows' max, then lse2
+    L.bars = L.fm + kEpiWarps * kRows * 4u;
+    L.total = L.bars + 256u;
+    return L;
+}
+
+// Barrier block (8-byte slots): q_full[2], q_empty[2], t_full[2], t_empty[2],
+// e_sync, drain, TMEM base word, abort word, k_full[4], k_empty[4].
+struct Bars {
+    uint32_t base;
+    __device__ __forceinline__ uint32_t q_full(int s) const { return base + 8u * s; }
+    __device__ __forceinline__ uint32_t q_empty(int s) const { return base + 16u + 8u * s; }
+    __device__ __forceinline__ uint32_t t_full(int s) const { return base + 32u + 8u * s; }
+    __device__ __forceinline__ uint32_t t_empty(int s) const { return base + 48u + 8u * s; }
+    __device__ __forceinline__ uint32_t e_sync() const { return base + 64u; }
+    __device__ __forceinline__ uint32_t drain() const { return base + 72u; }
+    __device__ __forceinline__ uint32_t tmem_slot() const { return base + 80u; }
+    __device__ __forceinline__ uint32_t abort() const { return base + 88u; }
+    __device__ __forceinline__ uint32_t k_full(int st) const { return base + 96u + 8u * st; }
+    __device__ __forceinline__ uint32_t k_empty(int st) const { return base + 128u + 8u * st; }
+};
+
+__device__ inline void raise_abort(const Bars& b, int* err)
+{
+    tc::st_shared_volatile(b.abort(), 1u);
+    if (err) atomicExch(err, tc::kErrTimeout);
+}
+
+__device__ inline void unit_range(int units, int* u0, int* u1)
+{
+    *u0 = (int)(((long long)blockIdx.x * units) / gridDim.x);
+    *u1 = (int)(((long long)(blockIdx.x + 1) * units) / gridDim.x);
+}
+
+// ---------------------------------------------------------------- producer
+
+template <int D>
+__device__ void produce(const TcArgs& a, const Layout& L, uint8_t* sm, const Bars& b)
+{
+    constexpr int H = D / 64;
+    const Shape& s = a.s;
+    const int lane = threadIdx.x & 31;
+    const int ntiles = (s.N + kTok - 1) / kTok;
+    int u0, u1;
+    unit_range(s.units, &u0, &u1);
+    int n = 0, kt = 0;
+    bool ok = true;
+    if (lane == 0) {
+        for (int u = u0; u < u1 && ok; ++u, ++n) {
+            const int pair = u / s.hkv, h = u - pair * s.hkv;
+            const int slot = n & 1, use = n >> 1;
+            if (!tc::mbar_wait(b.q_empty(slot), (use & 1) ^ 1, b.abort())) { ok = false; break; }
+            tc::mbar_arrive_expect_tx(b.q_full(slot), L.q_slot);
+            for (int kh = 0; kh < H; ++kh)
+                tc::tma_load_2d(sm + L.q + slot * L.q_slot + kh * L.q_half, a.qmaps + pair, kh * 64,
+                                h * s.rows, b.q_full(slot));
+            for (int t = 0; t < ntiles; ++t, ++kt) {
+                const int st = kt % kStages, m = kt / kStages;
+                if (!tc::mbar_wait(b.k_empty(st), (m & 1) ^ 1, b.abort())) { ok = false; break; }
+                tc::mbar_arrive_expect_tx(b.k_full(st), L.k_stage);
+                for (int kh = 0; kh < H; ++kh)
+                    tc::tma_load_2d(sm + L.k + st * L.k_stage + kh * kTok * 128, a.kmaps + pair,
+                                    kh * 64, h * s.N + t * kTok, b.k_full(st));
+            }
+        }
+        if (!ok) raise_abort(b, a.err);
+        // the last load of every stage and slot must land before the CTA exits
+        for (int st = 0; st < kStages && st < kt; ++st) {
+            const int last = kt - 1 - ((kt - 1 - st) % kStages);
+            tc::mbar_wait(b.k_full(st), (last / kStages) & 1, 0u);
+        }
+        for (int slot = 0; slot < 2 && slot < n; ++slot) {
+            const int last = n - 1 - ((n - 1 - slot) & 1);
+            tc::mbar_wait(b.q_full(slot), (last >> 1) & 1, 0u);
+        }
+    }
+}
+
+// ------------------------------------------------------------- MMA issuer
+
+template <int D>
+__device__ void issue(const TcArgs& a, const Layout& L, uint8_t* sm, const Bars& b)
+{
+    const Shape& s = a.s;
+    const int ntiles = (s.N + kTok - 1) / kTok;
+    const uint32_t tmem = tc::ld_shared(b.tmem_slot());
+    const uint32_t sbase = smem_u32(sm);
+    const uint32_t idesc = tc::idesc_bf16(kTok, kRows);
+    int u0, u1;
+    unit_range(s.units, &u0, &u1);
+    int n = 0, kt = 0;
+    bool ok = true;
+    for (int u = u0; u < u1 && ok; ++u, ++n) {
+        const int slot = n & 1, use = n >> 1;
+        if (!tc::mbar_wait(b.q_full(slot), use & 1, b.abort()) ||
+            !tc::mbar_wait(b.t_empty(slot), (use & 1) ^ 1, b.abort())) {
+            ok = false;
+            break;
+        }
+        tc::fence_after_sync();
+        const uint32_t qaddr = sbase + L.q + slot * L.q_slot;
+        for (int t = 0; t < ntiles; ++t, ++kt) {
+            const int st = kt % kStages, m = kt / kStages;
+            if (!tc::mbar_wait(b.k_full(st), m & 1, b.abort())) { ok = false; break; }
+            tc::fence_after_sync();
+            const uint32_t kaddr = sbase + L.k + st * L.k_stage;
+            const uint32_t d_tmem = tmem + slot * kSlotCols + t * kRows;
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+                const int kh = kk / 4;
+                const uint32_t koff = (kk % 4) * 32;
+                tc::umma_bf16(d_tmem, tc::sdesc_sw128(kaddr + kh * kTok * 128 + koff),
+                              tc::sdesc_sw128(qaddr + kh * L.q_half + koff), idesc, kk > 0);
+            }
+            tc::umma_commit(b.k_empty(st));
+        }
+        if (!ok) break;
+        tc::umma_commit(b.t_full(slot));   // the unit's logits are complete
+        tc::umma_commit(b.q_empty(slot));  // and its window rows may be replaced
+    }
+    if (!ok) raise_abort(b, a.err);
+    tc::umma_commit(b.drain());
+    tc::mbar_wait(b.drain(), 0, 0u);
+}
+
+// ---------------------------------------------------------------- epilogue
+
+// After the call, lane l of the warp holds op over the warp's 32 lanes of
+// v[l] (a butterfly transpose: 31 shuffles for 32 values).
+template <bool MAX>
+__device__ __forceinline__ float transpose_reduce(float* v)
+{
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int w = 16; w >= 1; w >>= 1) {
+        const bool upper = (lane & w) != 0;
+#pragma unroll
+        for (int j = 0; j < w; ++j) {
+            const float send = upper ? v[j] : v[j + w];
+            const float keep = upper ? v[j + w] : v[j];
+            const float recv = __shfl_xor_sync(0xffffffffu, send, w);
+            v[j] = MAX ? fmaxf(keep, recv) : keep + recv;
+        }
+    }
+    return v[0];
+}
+
+// Logits of one tile for this thread's token (its TMEM lane), scaled by c;
+// rows the token is hidden from are -inf: padding rows (bit r of `real` is
+// clear), tokens past N, and, in tiles that reach into the window, the rows
+// whose position precedes the token (row r sits at N - W + r mod W).
+__device__ __forceinline__ void load_row_logits(uint32_t taddr, const Shape& s, int tile, int tok,
+                                                float c, uint32_t real, float* v)
+{
+    tc::tmem_ld32(taddr, v);
+    tc::tmem_ld_wait_regs32(v);
+    if (tile * kTok + kTok - 1 <= s.N - s.W) {  // whole tile before the window: no mask
+#pragma unroll
+        for (int r = 0; r < kRows; ++r) v[r] = (real >> r) & 1u ? v[r] * c : -INFINITY;
+        return;
+    }
+    const int lim = tok < s.N ? tok - (s.N - s.W) : s.W;  // rows with r mod W < lim are hidden
+    int rm = 0;                                            // r mod W
+#pragma unroll
+    for (int r = 0; r < kRows; ++r) {
+        v[r] = ((real >> r) & 1u) && rm >= lim ? v[r] * c : -INFINITY;
+        rm = rm + 1 == s.W ? 0 : rm + 1;
+    }
+}
+
+__device__ __forceinline__ bool epi_sync(const Bars& b, int& nsync)
+{
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) tc::mbar_arrive(b.e_sync());
+    const bool ok = tc::mbar_wait(b.e_sync(), nsync & 1, b.abort());
+    ++nsync;
+    return ok;
+}
+
+template <int D>
+__device__ void epilogue(const TcArgs& a, const Layout& L, uint8_t* sm, const Bars& b)
+{
+    const Shape& s = a.s;
+    const int ntiles = (s.N + kTok - 1) / kTok;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int ew = warp - 2;               // epilogue warp 0..15
+    const int quarter = warp & 3;          // TMEM lanes this warp may access
+    const int group = ew >> 2;             // tiles t = group mod kGroups
+    const uint32_t tl = tc::ld_shared(b.tmem_slot()) + ((uint32_t)(quarter * 32) << 16);
+    float* xr = reinterpret_cast<float*>(sm + L.xr);
+    float* xs = reinterpret_cast<float*>(sm + L.xs);
+    float* fm = reinterpret_cast<float*>(sm + L.fm) + ew * kRows;  // this warp's copy
+    const float c = kLog2e * rsqrtf((float)D);
+    const float log2_gw = log2f((float)s.rows);
+    // bit r: row r is a window row / a last-position row (r mod W = W - 1)
+    uint32_t real = 0u, last = 0u;
+    for (int r = 0; r < kRows && r < s.rows; ++r) {
+        real |= 1u << r;
+        if (r % s.W == s.W - 1) last |= 1u << r;
+    }
+    int u0, u1;
+    unit_range(s.units, &u0, &u1);
+    int n = 0, nsync = 0;
+    bool ok = true;
+    for (int u = u0; u < u1 && ok; ++u, ++n) {
+        const int slot = n & 1, use = n >> 1;
+        if (!tc::mbar_wait(b.t_full(slot), use & 1, b.abort())) { ok = false; break; }
+        tc::fence_after_sync();
+        const uint32_t tbase = tl + slot * kSlotCols;
+        // (1) each row's maximum over the unit's tokens
+        float v[kRows], acc[kRows];
+#pragma unroll
+        for (int r = 0; r < kRows; ++r) acc[r] = -INFINITY;
+        for (int t = group; t < ntiles; t += kGroups) {
+            load_row_logits(tbase + t * kRows, s, t, t * kTok + quarter * 32 + lane, c, real, v);
+#pragma unroll
+            for (int r = 0; r < kRows; ++r) acc[r] = fmaxf(acc[r], v[r]);
+        }
+        xr[ew * kRows + lane] = transpose_reduce<true>(acc);
+        if (!epi_sync(b, nsync)) { ok = false; break; }
+        float mrow = -INFINITY;
+        for (int w = 0; w < kEpiWarps; ++w) mrow = fmaxf(mrow, xr[w * kRows + lane]);
+        fm[lane] = mrow == -INFINITY ? 0.f : mrow;
+        __syncwarp();
+        // (2) each row's sum of 2^(x - max)
+#pragma unroll
+        for (int r = 0; r < kRows; ++r) acc[r] = 0.f;
+        for (int t = group; t < ntiles; t += kGroups) {
+            load_row_logits(tbase + t * kRows, s, t, t * kTok + quarter * 32 + lane, c, real, v);
+#pragma unroll
+            for (int r = 0; r < kRows; ++r) acc[r] += v[r] == -INFINITY ? 0.f : fast_exp2(v[r] - fm[r]);
+        }
+        xs[ew * kRows + lane] = transpose_reduce<false>(acc);
+        if (!epi_sync(b, nsync)) { ok = false; break; }
+        float z = 0.f;
+        for (int w = 0; w < kEpiWarps; ++w) z += xs[w * kRows + lane];
+        // log2 of the normaliser plus log2(G W): a share is then A / (G W)
+        fm[lane] = fm[lane] + log2f(z) + log2_gw;
+        __syncwarp();
+        // (3) the token's B (all rows), Q (last-position rows) and E
+        for (int t = group; t < ntiles; t += kGroups) {
+            const int tok = t * kTok + quarter * 32 + lane;
+            load_row_logits(tbase + t * kRows, s, t, tok, c, real, v);
+            float bsum = 0.f, qsum = 0.f;
+#pragma unroll
+            for (int r = 0; r < kRows; ++r) {
+                // hidden tokens and padding rows (whose normaliser is -inf) add nothing
+                const float x = v[r] == -INFINITY ? 0.f : fast_exp2(v[r] - fm[r]);
+                bsum += x;
+                if ((last >> r) & 1u) qsum += x;
+            }
+            qsum *= (float)s.W;
+            if (tok < s.N) {
+                const size_t idx = (size_t)u * s.N + tok;
+                a.B[idx] = bsum;
+                a.Q[idx] = qsum;
+                a.E[idx] = fmaxf(qsum - bsum, 0.f);
+            }
+        }
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(b.t_empty(slot));  // this unit's TMEM half is read
+    }
+    if (!ok) raise_abort(b, a.err);
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1) window_onepass_kernel(TcArgs a)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    const Layout L = layout<D>();
+    Bars b;
+    b.base = smem_u32(sm + L.bars);
+    const int warp = threadIdx.x >> 5;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < 2; ++i) {
+            tc::mbar_init(b.q_full(i), 1);
+            tc::mbar_init(b.q_empty(i), 1);
+            tc::mbar_init(b.t_full(i), 1);
+            tc::mbar_init(b.t_empty(i), kEpiWarps);  // one arrival per epilogue warp
+        }
+        for (int i = 0; i < kStages; ++i) {
+            tc::mbar_init(b.k_full(i), 1);
+            tc::mbar_init(b.k_empty(i), 1);
+        }
+        tc::mbar_init(b.e_sync(), kEpiWarps);
+        tc::mbar_init(b.drain(), 1);
+        tc::st_shared_volatile(b.abort(), 0u);
+        tc::fence_barrier_init();
+    }
+    if (warp == 1) {
+        tc::tmem_alloc(b.tmem_slot(), 512);
+        tc::tmem_relinquish();
+    }
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+
+    if (warp == 0)
+        produce<D>(a, L, sm, b);
+    else if (warp == 1) {
+        if (tc::elect_one()) issue<D>(a, L, sm, b);
+    } else {
+        epilogue<D>(a, L, sm, b);
+    }
+
+    tc::fence_before_sync();
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tc::fence_after_sync();
+        tc::tmem_dealloc(tc::ld_shared(b.tmem_slot()), 512);
+    }
+}
+
+int num_sms_onepass()
+{
+    int dev = 0, n = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    return n > 0 ? n : 1;
+}
+
+template <int D>
+cudaError_t launch_d(const TcArgs& a, cudaStream_t st)
+{
+    const Layout L = layout<D>();
+    size_t bytes = L.total + 1024;
+    if (bytes < 116 * 1024) bytes = 116 * 1024;  // one CTA (one TMEM allocation) per SM
+    cudaError_t e = cudaFuncSetAttribute(window_onepass_kernel<D>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e != cudaSuccess) return e;
+    const int sms = num_sms_onepass();
+    const int grid = a.s.units < sms ? a.s.units : sms;
+    window_onepass_kernel<D><<<grid, kThreads, bytes, st>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+bool window_onepass_fits(const Shape& s)
+{
+    return s.rows <= kRows && (s.d == 64 || s.d == 128) && (s.N + kTok - 1) / kTok <= kMaxTiles;
+}
+
+cudaError_t launch_window_onepass(const TcArgs& a, cudaStream_t st)
+{
+    if (!window_onepass_fits(a.s)) return cudaErrorInvalidValue;
+    return a.s.d == 128 ? launch_d<128>(a, st) : launch_d<64>(a, st);
+}
+
+}  // namespace bacon

@@ -34,6 +34,12 @@ cudaError_t launch_window_scores_tc(const TcArgs& a, cudaStream_t st);
 cudaError_t launch_window_combine(const Shape& s, int chunks, const float2* partial, float* lse2,
                                   cudaStream_t st);
 
+// One pass over K for units whose logits fit in tensor memory (at most 32
+// window rows and 1024 tokens): B, Q and E as the two passes give them,
+// without the partial statistics or the merge.
+bool window_onepass_fits(const Shape& s);
+cudaError_t launch_window_onepass(const TcArgs& a, cudaStream_t st);
+
 // Per (request, layer) natural-log softmax normalisers of the window rows,
 // [Hq][W] fp32, as a prefill attention kernel produces them.
 struct LseTable {
