@@ -14,7 +14,9 @@ on work lists cut the way the kernels cut them (each CTA a contiguous range
 of 1024-token chunks over (request, layer, kv-head) units), and checks that
 every schedule finishes and every wait returns in its own phase.  The
 variant in which the merging group does not first wait for the slot's
-previous read (the kernels' earlier protocol) fails the check.
+previous read (the kernels' earlier protocol) fails the check.  The one-pass
+kernel (logits resident in TMEM, two CTA-wide syncs per unit) is modelled
+the same way.
 """
 
 import random
@@ -212,3 +214,102 @@ def test_model_catches_the_unguarded_merger():
     chunks = cta_range(3, 2, 1, 0)
     faults = [simulate(chunks, 11, 8, 1, 4, 4, 1, True, False, s) for s in range(8)]
     assert any(f is not None for f in faults)
+
+
+# ------------------------------------------------ one-pass kernel
+
+def simulate_onepass(n_units, ntiles, stages, epi_warps, seed):
+    """The one-pass kernel: a unit's logits occupy one of two TMEM halves;
+    the epilogue warps meet twice per unit at a CTA-wide mbarrier and reuse
+    two shared-memory buffers of partials (row maxima, row sums)."""
+    rnd = random.Random(seed)
+    k_full = [Bar(1, f"k_full{i}") for i in range(stages)]
+    k_empty = [Bar(1, f"k_empty{i}") for i in range(stages)]
+    q_full = [Bar(1, f"q_full{i}") for i in range(2)]
+    q_empty = [Bar(1, f"q_empty{i}") for i in range(2)]
+    t_full = [Bar(1, f"t_full{i}") for i in range(2)]
+    t_empty = [Bar(epi_warps, f"t_empty{i}") for i in range(2)]
+    e_sync = Bar(epi_warps, "e_sync")
+    drain = Bar(1, "drain")
+    tma, commits = [], []
+    xr, xs = {}, {}
+
+    def producer():
+        kt = 0
+        for n in range(n_units):
+            yield from wait(q_empty[n & 1], (n >> 1) - 1)
+            tma.append(q_full[n & 1])
+            for _ in range(ntiles):
+                st, m = kt % stages, kt // stages
+                yield from wait(k_empty[st], m - 1)
+                tma.append(k_full[st])
+                kt += 1
+                yield
+
+    def mma():
+        kt = 0
+        for n in range(n_units):
+            yield from wait(q_full[n & 1], n >> 1)
+            yield from wait(t_empty[n & 1], (n >> 1) - 1)
+            for _ in range(ntiles):
+                st, m = kt % stages, kt // stages
+                yield from wait(k_full[st], m)
+                kt += 1
+                yield
+                commits.append(k_empty[st])
+            commits.append(t_full[n & 1])
+            commits.append(q_empty[n & 1])
+        commits.append(drain)
+        yield from wait(drain, 0)
+
+    def epilogue(w):
+        nsync = 0
+        for n in range(n_units):
+            yield from wait(t_full[n & 1], n >> 1)
+            xr[w] = n
+            yield
+            e_sync.arrive()
+            yield from wait(e_sync, nsync)
+            nsync += 1
+            if any(xr[v] != n for v in range(epi_warps)):
+                raise Fault(f"row maxima of unit {n} overwritten before they were read")
+            xs[w] = n
+            yield
+            e_sync.arrive()
+            yield from wait(e_sync, nsync)
+            nsync += 1
+            if any(xs[v] != n for v in range(epi_warps)):
+                raise Fault(f"row sums of unit {n} overwritten before they were read")
+            yield
+            t_empty[n & 1].arrive()
+
+    procs = [producer(), mma()] + [epilogue(w) for w in range(epi_warps)]
+    live = list(range(len(procs)))
+    for _ in range(300000):
+        if not live and not tma and not commits:
+            return None
+        r = rnd.random()
+        if tma and r < 0.25:
+            tma.pop(rnd.randrange(len(tma))).arrive()
+            continue
+        if commits and r < 0.5:
+            commits.pop(0).arrive()
+            continue
+        if not live:
+            continue
+        i = rnd.choice(live)
+        try:
+            next(procs[i])
+        except StopIteration:
+            live.remove(i)
+        except Fault as f:
+            return str(f)
+    return "deadlock"
+
+
+@pytest.mark.parametrize("n_units,ntiles,stages", [(1, 1, 4), (3, 5, 2), (7, 8, 4), (9, 8, 3),
+                                                   (6, 1, 4), (4, 7, 3)])
+def test_onepass_protocol(n_units, ntiles, stages):
+    for seed in range(6):
+        fault = simulate_onepass(n_units, ntiles, stages, 8, seed)
+        assert fault is None, (seed, fault)
