@@ -15,9 +15,10 @@
 //   * eight epilogue warps (two groups x four lane quarters; group g takes
 //     the tiles t = g mod 2) reduce each row's maximum over their tokens by a
 //     butterfly transpose across the warp's lanes, meet at a CTA-wide
-//     mbarrier, reduce the sums of 2^(x - max) the same way, meet again, and
-//     then each thread sums its token's shares over the rows (B), over the
-//     last-position rows (Q) and stores E = [Q - B]_+.
+//     mbarrier, write p = 2^(x - max) over the logits in TMEM while reducing
+//     the rows' sums of p the same way, meet again, and then each thread
+//     scales its token's p by 1 / (row sum x G W) and sums them over the rows
+//     (B) and over the last-position rows (Q), and stores E = [Q - B]_+.
 // Every wait is bounded (abort flag, clock limit): on timeout the CTA records
 // BACON_ETIMEOUT, drains its own copies and MMAs, frees TMEM and returns.
 #include <cuda_bf16.h>
@@ -57,12 +58,12 @@ __host__ __device__ inline Layout layout()
     L.xs = L.xr + kEpiWarps * kRows * 4u;          // [warp][row] partial sums
     L.fm = L.xs + kEpiWarps * kRows * 4u;          // [warp][row] the rows' max, then lse2
     L.bars = L.fm + kEpiWarps * kRows * 4u;
-    L.total = L.bars + 256u;
+    L.total = L.bars + 96u + 16u * kStages;
     return L;
 }
 
 // Barrier block (8-byte slots): q_full[2], q_empty[2], t_full[2], t_empty[2],
-// e_sync, drain, TMEM base word, abort word, k_full[4], k_empty[4].
+// e_sync, drain, TMEM base word, abort word, k_full[kStages], k_empty[kStages].
 struct Bars {
     uint32_t base;
     __device__ __forceinline__ uint32_t q_full(int s) const { return base + 8u * s; }
@@ -74,7 +75,10 @@ struct Bars {
     __device__ __forceinline__ uint32_t tmem_slot() const { return base + 80u; }
     __device__ __forceinline__ uint32_t abort() const { return base + 88u; }
     __device__ __forceinline__ uint32_t k_full(int st) const { return base + 96u + 8u * st; }
-    __device__ __forceinline__ uint32_t k_empty(int st) const { return base + 128u + 8u * st; }
+    __device__ __forceinline__ uint32_t k_empty(int st) const
+    {
+        return base + 96u + 8u * (kStages + st);
+    }
 };
 
 __device__ inline void raise_abort(const Bars& b, int* err)
@@ -248,7 +252,6 @@ __device__ void epilogue(const TcArgs& a, const Layout& L, uint8_t* sm, const Ba
     float* xs = reinterpret_cast<float*>(sm + L.xs);
     float* fm = reinterpret_cast<float*>(sm + L.fm) + ew * kRows;  // this warp's copy
     const float c = kLog2e * rsqrtf((float)D);
-    const float log2_gw = log2f((float)s.rows);
     // bit r: row r is a window row / a last-position row (r mod W = W - 1)
     uint32_t real = 0u, last = 0u;
     for (int r = 0; r < kRows && r < s.rows; ++r) {
@@ -279,30 +282,36 @@ __device__ void epilogue(const TcArgs& a, const Layout& L, uint8_t* sm, const Ba
         for (int w = 0; w < kEpiWarps; ++w) mrow = fmaxf(mrow, xr[w * kRows + lane]);
         fm[lane] = mrow == -INFINITY ? 0.f : mrow;
         __syncwarp();
-        // (2) each row's sum of 2^(x - max)
+        // (2) each row's sum of p = 2^(x - max); p replaces the logit in TMEM
+        // (hidden tokens and padding rows give p = 0)
 #pragma unroll
         for (int r = 0; r < kRows; ++r) acc[r] = 0.f;
         for (int t = group; t < ntiles; t += kGroups) {
             load_row_logits(tbase + t * kRows, s, t, t * kTok + quarter * 32 + lane, c, real, v);
 #pragma unroll
-            for (int r = 0; r < kRows; ++r) acc[r] += v[r] == -INFINITY ? 0.f : fast_exp2(v[r] - fm[r]);
+            for (int r = 0; r < kRows; ++r) {
+                v[r] = v[r] == -INFINITY ? 0.f : fast_exp2(v[r] - fm[r]);
+                acc[r] += v[r];
+            }
+            tc::tmem_st32(tbase + t * kRows, v);
         }
+        tc::tmem_st_wait();
         xs[ew * kRows + lane] = transpose_reduce<false>(acc);
         if (!epi_sync(b, nsync)) { ok = false; break; }
         float z = 0.f;
         for (int w = 0; w < kEpiWarps; ++w) z += xs[w * kRows + lane];
-        // log2 of the normaliser plus log2(G W): a share is then A / (G W)
-        fm[lane] = fm[lane] + log2f(z) + log2_gw;
+        // a token's share of row r is p / (Z_r G W) (= A / (G W)); padding rows 0
+        fm[lane] = z > 0.f ? 1.f / (z * (float)s.rows) : 0.f;
         __syncwarp();
         // (3) the token's B (all rows), Q (last-position rows) and E
         for (int t = group; t < ntiles; t += kGroups) {
             const int tok = t * kTok + quarter * 32 + lane;
-            load_row_logits(tbase + t * kRows, s, t, tok, c, real, v);
+            tc::tmem_ld32(tbase + t * kRows, v);
+            tc::tmem_ld_wait_regs32(v);
             float bsum = 0.f, qsum = 0.f;
 #pragma unroll
             for (int r = 0; r < kRows; ++r) {
-                // hidden tokens and padding rows (whose normaliser is -inf) add nothing
-                const float x = v[r] == -INFINITY ? 0.f : fast_exp2(v[r] - fm[r]);
+                const float x = v[r] * fm[r];
                 bsum += x;
                 if ((last >> r) & 1u) qsum += x;
             }
