@@ -26,7 +26,8 @@ def _rank(rank, world, port, out):
 def test_replicas_use_the_slowest_rank():
     world = 2
     port = 29500 + (os.getpid() % 2000)
-    out = mp.Manager().dict()
+    # the result dict's server process is spawned too: nothing is forked
+    out = mp.get_context("spawn").Manager().dict()
     mp.spawn(_rank, args=(world, port, out), nprocs=world, join=True)
     assert out[0] == out[1]
     slowest, value = out[0]
