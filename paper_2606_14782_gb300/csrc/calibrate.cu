@@ -19,12 +19,14 @@ namespace {
 
 using namespace sel;
 
-// At most kMaxPer tokens per thread.  Threads per CTA depend on the prompt
-// length only (so that every call on the same shape reduces in the same
-// order and gives the same bits): 256 up to 2048 tokens, where several CTAs
-// share an SM, else 1024.
+// Threads per CTA and tokens per thread depend on the prompt length only
+// (so that every call on the same shape reduces in the same order and gives
+// the same bits): 256 threads of up to 8 tokens up to 2048 tokens, where
+// several CTAs share an SM; 1024 threads of up to 16 tokens up to 16384
+// tokens; 1024 threads of up to kMaxPer tokens above.
 constexpr int kMaxPer = 24;
 constexpr int kSmallPrompt = 2048;
+constexpr int kMidPrompt = 16384;  // 1024 threads x 16 tokens
 
 // Block-wide fp32 sum by a shuffle tree (pairwise, so the rounding error
 // grows with log2 of the count).  FP64 is avoided: its rate on this part is
@@ -79,6 +81,14 @@ __device__ float4 block_sum4(float4 v, float* red)
     return tot;
 }
 
+// Ask L2 to fetch the n floats at p (one prefetch per 128-byte line, every
+// address inside the array), so that later loads of them hit L2.
+__device__ __forceinline__ void prefetch_l2(const float* p, int n)
+{
+    for (int i = (int)threadIdx.x * 32; i < n; i += (int)blockDim.x * 32)
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(p + i));
+}
+
 // dst[0, n) = src[0, n) with independent 16-byte loads (n % 4 == 0 and both
 // 16-byte aligned), so the copy costs a few memory round trips, not one per
 // element.
@@ -100,6 +110,8 @@ __device__ __forceinline__ void stage(float* dst, const float* src, int n)
 
 // One unit (request, layer, kv-head) u under hyper-parameters c.  lam_out
 // (may be null) receives lambda; idx_pair is the pair's [Hkv][kept] output.
+// PER bounds the tokens per thread (N <= PER blockDim.x).
+template <int PER>
 __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, const CalibArgs& a,
                                                int u, float* lam_out, int32_t* idx_pair)
 {
@@ -133,6 +145,11 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
         const int half = c.pool / 2;
         const int nprev = min(c.m, layer);
         const float inv_prev = nprev > 0 ? 1.f / (float)nprev : 0.f;
+        // the residuals of this layer and of the preceding ones are read
+        // only after the pooling: start bringing them into L2 now
+        prefetch_l2(Ec, N);
+        if (c.use_T)
+            for (int j = layer - nprev; j < layer; ++j) prefetch_l2(Eof(j), N);
         // B -> Vs (staging), then the pooled backbone over the candidates -> Sb
         if ((N & 3) == 0)
             stage(Vs, Bu, N);
@@ -145,6 +162,7 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
             if (i < n_cand) {
                 mx = -INFINITY;
                 const int lo = max(0, i - half), hi = min(n_cand - 1, i + half);
+#pragma unroll 4
                 for (int v = lo; v <= hi; ++v) mx = fmaxf(mx, Vs[v]);
                 kmin = min(kmin, float_key(mx));
                 kmax = max(kmax, float_key(mx));
@@ -158,27 +176,32 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
         else
             for (int i = threadIdx.x; i < N; i += blockDim.x) Vs[i] = Ec[i];
         __syncthreads();
-        float vreg[kMaxPer];
+        float vreg[PER];
         // persistence: mean of E over the preceding min(m, l) layers (Eqs. 8-9)
 #pragma unroll
-        for (int k = 0; k < kMaxPer; ++k) vreg[k] = 0.f;
+        for (int k = 0; k < PER; ++k) vreg[k] = 0.f;
         if (c.use_T) {
             for (int j = layer - nprev; j < layer; ++j) {
                 const float* Ej = Eof(j);
+                // every load in flight at once: indices past the end are
+                // clamped to the last token (in bounds) and their values
+                // dropped
+                float x[PER];
 #pragma unroll
-                for (int k = 0; k < kMaxPer; ++k) {
-                    const int i = threadIdx.x + k * blockDim.x;
-                    if (i < N) vreg[k] += Ej[i];
-                }
+                for (int k = 0; k < PER; ++k) x[k] = Ej[min((int)threadIdx.x + k * (int)blockDim.x, N - 1)];
+#pragma unroll
+                for (int k = 0; k < PER; ++k)
+                    if ((int)threadIdx.x + k * (int)blockDim.x < N) vreg[k] += x[k];
             }
         }
 #pragma unroll
-        for (int k = 0; k < kMaxPer; ++k) {
+        for (int k = 0; k < PER; ++k) {
             const int i = threadIdx.x + k * blockDim.x;
             if (i < N) {
                 // coherence: truncated radius-r box mean of E (Eqs. 5-7)
                 const int lo = max(0, i - c.r), hi = min(N - 1, i + c.r);
                 float sum = 0.f;
+#pragma unroll 4
                 for (int v = lo; v <= hi; ++v) sum += Vs[v];
                 const float L = sum / (float)(hi - lo + 1);
                 float V = 0.f;
@@ -191,7 +214,7 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
         __syncthreads();
         float vsum = 0.f;  // over the candidates: the shift of the moments below
 #pragma unroll
-        for (int k = 0; k < kMaxPer; ++k) {
+        for (int k = 0; k < PER; ++k) {
             const int i = threadIdx.x + k * blockDim.x;
             if (i < N) Vs[i] = vreg[k];
             if (i < n_cand) vsum += vreg[k];
@@ -281,25 +304,25 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
     for (int w = threadIdx.x; w < win; w += blockDim.x) out[keep + w] = N - W + w;
 }
 
-template <int T>
+template <int T, int PER>
 __global__ void __launch_bounds__(T, 1024 / T)
 calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
 {
     const int u = blockIdx.x;
-    calibrate_unit(s, c, a, u, a.lambda + u, a.idx[u / s.hkv]);
+    calibrate_unit<PER>(s, c, a, u, a.lambda + u, a.idx[u / s.hkv]);
 }
 
 // Several hyper-parameter sets over the same B and residuals: CTA (u, v)
 // runs unit u under variant v; variant v's indices start v *
 // idx_variant_stride elements after the single-variant layout and its
 // lambdas v * units after a.lambda.
-template <int T>
+template <int T, int PER>
 __global__ void __launch_bounds__(T, 1024 / T)
 calibrate_sweep_kernel(Shape s, CalibTable t, CalibArgs a)
 {
     const int u = blockIdx.x, v = blockIdx.y;
     float* lam = a.lambda ? a.lambda + (size_t)v * s.units + u : nullptr;
-    calibrate_unit(s, t.c[v], a, u, lam, a.idx[u / s.hkv] + (size_t)v * a.idx_variant_stride);
+    calibrate_unit<PER>(s, t.c[v], a, u, lam, a.idx[u / s.hkv] + (size_t)v * a.idx_variant_stride);
 }
 
 }  // namespace
@@ -308,26 +331,26 @@ size_t calibrate_smem(int N) { return (size_t)2 * N * sizeof(float); }
 
 namespace {
 
-template <int T>
+template <int T, int PER>
 cudaError_t launch_select_t(const Shape& s, const Calib& c, const CalibArgs& a, cudaStream_t st)
 {
     const size_t sm = calibrate_smem(s.N);
-    cudaError_t e = cudaFuncSetAttribute(calibrate_select_kernel<T>,
+    cudaError_t e = cudaFuncSetAttribute(calibrate_select_kernel<T, PER>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
-    calibrate_select_kernel<T><<<s.units, T, sm, st>>>(s, c, a);
+    calibrate_select_kernel<T, PER><<<s.units, T, sm, st>>>(s, c, a);
     return cudaGetLastError();
 }
 
-template <int T>
+template <int T, int PER>
 cudaError_t launch_sweep_t(const Shape& s, const CalibTable& t, int variants, const CalibArgs& a,
                            cudaStream_t st)
 {
     const size_t sm = calibrate_smem(s.N);
-    cudaError_t e = cudaFuncSetAttribute(calibrate_sweep_kernel<T>,
+    cudaError_t e = cudaFuncSetAttribute(calibrate_sweep_kernel<T, PER>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
-    calibrate_sweep_kernel<T><<<dim3(s.units, variants), T, sm, st>>>(s, t, a);
+    calibrate_sweep_kernel<T, PER><<<dim3(s.units, variants), T, sm, st>>>(s, t, a);
     return cudaGetLastError();
 }
 
@@ -336,15 +359,17 @@ cudaError_t launch_sweep_t(const Shape& s, const CalibTable& t, int variants, co
 cudaError_t launch_calibrate_select(const Shape& s, const Calib& c, const CalibArgs& a,
                                     cudaStream_t st)
 {
-    return s.N <= kSmallPrompt ? launch_select_t<256>(s, c, a, st)
-                               : launch_select_t<1024>(s, c, a, st);
+    if (s.N <= kSmallPrompt) return launch_select_t<256, kSmallPrompt / 256>(s, c, a, st);
+    if (s.N <= kMidPrompt) return launch_select_t<1024, kMidPrompt / 1024>(s, c, a, st);
+    return launch_select_t<1024, kMaxPer>(s, c, a, st);
 }
 
 cudaError_t launch_calibrate_sweep(const Shape& s, const CalibTable& t, int variants,
                                    const CalibArgs& a, cudaStream_t st)
 {
-    return s.N <= kSmallPrompt ? launch_sweep_t<256>(s, t, variants, a, st)
-                               : launch_sweep_t<1024>(s, t, variants, a, st);
+    if (s.N <= kSmallPrompt) return launch_sweep_t<256, kSmallPrompt / 256>(s, t, variants, a, st);
+    if (s.N <= kMidPrompt) return launch_sweep_t<1024, kMidPrompt / 1024>(s, t, variants, a, st);
+    return launch_sweep_t<1024, kMaxPer>(s, t, variants, a, st);
 }
 
 }  // namespace bacon

@@ -107,6 +107,7 @@ __device__ void produce(const TcArgs& a, const Layout& L, uint8_t* sm, const Bar
     int n = 0, kt = 0;
     bool ok = true;
     if (lane == 0) {
+        const uint64_t kpol = tc::l2_evict_first_policy();  // K is read once
         for (int u = u0; u < u1 && ok; ++u, ++n) {
             const int pair = u / s.hkv, h = u - pair * s.hkv;
             const int slot = n & 1, use = n >> 1;
@@ -120,8 +121,8 @@ __device__ void produce(const TcArgs& a, const Layout& L, uint8_t* sm, const Bar
                 if (!tc::mbar_wait(b.k_empty(st), (m & 1) ^ 1, b.abort())) { ok = false; break; }
                 tc::mbar_arrive_expect_tx(b.k_full(st), L.k_stage);
                 for (int kh = 0; kh < H; ++kh)
-                    tc::tma_load_2d(sm + L.k + st * L.k_stage + kh * kTok * 128, a.kmaps + pair,
-                                    kh * 64, h * s.N + t * kTok, b.k_full(st));
+                    tc::tma_load_2d_hint(sm + L.k + st * L.k_stage + kh * kTok * 128, a.kmaps + pair,
+                                         kh * 64, h * s.N + t * kTok, b.k_full(st), kpol);
             }
         }
         if (!ok) raise_abort(b, a.err);

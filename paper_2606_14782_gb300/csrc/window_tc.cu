@@ -223,6 +223,7 @@ __device__ __forceinline__ void produce(const TcArgs& a, const Smem& L, uint8_t*
     chunk_range(a.total_chunks, &c0, &c1);
     int cur_u = -1, qloads = 0, kt = 0;
     bool ok = true;
+    const uint64_t kpol = tc::l2_evict_first_policy();  // K is read once per pass
     for (int g = c0; g < c1 && ok; ++g) {
         const int u = g / a.chunks, ci = g - u * a.chunks;
         const int pair = u / s.hkv, h = u - pair * s.hkv;
@@ -254,8 +255,9 @@ __device__ __forceinline__ void produce(const TcArgs& a, const Smem& L, uint8_t*
                 if (!tc::mbar_wait(b.k_empty(st), (n & 1) ^ 1, b.abort())) { ok = false; break; }
                 tc::mbar_arrive_expect_tx(b.k_full(st), L.k_stage);
                 for (int kh = 0; kh < H; ++kh)
-                    tc::tma_load_2d(sm + L.k + st * L.k_stage + kh * kTileTok * 128, a.kmaps + pair,
-                                    kh * 64, h * s.N + t * kTileTok, b.k_full(st));
+                    tc::tma_load_2d_hint(sm + L.k + st * L.k_stage + kh * kTileTok * 128,
+                                         a.kmaps + pair, kh * 64, h * s.N + t * kTileTok,
+                                         b.k_full(st), kpol);
             }
         }
         ok = __shfl_sync(0xffffffffu, ok, 0);
