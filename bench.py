@@ -47,6 +47,9 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extras", action="store_true",
                     help="skip the prefill-normaliser and ablation-sweep measurements")
+    ap.add_argument("--record-traffic", metavar="NCU_CSV", default=None,
+                    help="store the DRAM bytes of an ncu --csv capture of this --config and "
+                         "--requests in profiles/traffic.json, then exit")
     return ap.parse_args()
 
 
@@ -138,16 +141,72 @@ def source_digest(names) -> str:
     return h.hexdigest()[:16]
 
 
-def kernel_traffic(kernel: str):
-    """DRAM bytes per launch from the committed ncu summary, or None when the
-    kernel's sources changed since the counters were taken."""
+# ncu kernel name -> (profile stage, the csrc files its code comes from)
+KERNEL_SOURCES = [
+    ("window_tc_kernel<", ", 1>", "window_stats", ["window_tc.cu", "window_tc.h", "tc.cuh", "common.cuh"]),
+    ("window_tc_kernel<", ", 2>", "window_scores", ["window_tc.cu", "window_tc.h", "tc.cuh", "common.cuh"]),
+    ("window_onepass_kernel", "", "window_scores",
+     ["window_onepass.cu", "window_tc.h", "tc.cuh", "common.cuh"]),
+    ("calibrate_select_kernel", "", "calibrate_select", ["calibrate.cu", "select.cuh", "common.cuh"]),
+    ("gather_kernel", "", "gather", ["gather.cu", "common.cuh"]),
+]
+
+
+def record_traffic(csv_path: str, workload: str, requests: int, command: str):
+    """Average dram__bytes_read.sum + dram__bytes_write.sum per launch of each
+    library kernel in an ncu --csv log, per request, into traffic.json."""
+    import csv
+    with open(csv_path) as f:
+        rows = list(csv.reader(line for line in f if not line.startswith("==")))
+    head = rows[0]
+    col = {name: i for i, name in enumerate(head)}
+    per_launch = {}
+    for r in rows[1:]:
+        if len(r) != len(head) or r[col["Metric Name"]] not in (
+                "dram__bytes_read.sum", "dram__bytes_write.sum"):
+            continue
+        unit = r[col["Metric Unit"]]
+        scale = {"byte": 1, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9}[unit]
+        key = (r[col["ID"]], r[col["Kernel Name"]])
+        per_launch[key] = per_launch.get(key, 0.0) + float(r[col["Metric Value"]].replace(",", "")) * scale
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
-            rec = json.load(f)[kernel]
+            rec = json.load(f)
+    except FileNotFoundError:
+        rec = {}
+    found = {}
+    for (_, name), b in per_launch.items():
+        for a, z, stage, srcs in KERNEL_SOURCES:
+            if a in name and z in name:
+                found.setdefault(stage, (srcs, []))[1].append(b)
+                break
+    for stage, (srcs, vals) in found.items():
+        rec.setdefault(workload, {})[stage] = {
+            "sources": srcs, "code_sha256_16": source_digest(srcs),
+            "dram_bytes_per_request": sum(vals) / len(vals) / requests,
+            "launches": len(vals),
+            "measured_on": f"{workload} workload, {requests} request(s): {command}; "
+                           "bench.py scales it by the requests of a launch (traffic grows in "
+                           "proportion to the (request, layer, kv-head) units processed)"}
+    with open(path, "w") as f:
+        json.dump(rec, f, indent=1)
+        f.write("\n")
+    return found
+
+
+def kernel_traffic(kernel: str, workload: str, requests: int):
+    """DRAM bytes per launch from the committed ncu summary of this kernel on
+    this workload (scaled to `requests`: traffic grows with the units), or
+    None when there is none or the kernel's sources changed since the
+    counters were taken."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)[workload][kernel]
         if source_digest(rec["sources"]) != rec["code_sha256_16"]:
             return None
-        return float(rec["dram_bytes_per_launch"])
+        return float(rec["dram_bytes_per_request"]) * requests
     except Exception:
         return None
 
@@ -236,6 +295,14 @@ def job_throughput(units_per_rank: int, world: int, ms: float) -> float:
 
 def main():
     args = parse()
+    if args.record_traffic:
+        from paper_2606_14782_gb300 import workloads
+        wl = workloads.CONFIGS[args.config]
+        req = args.requests or wl.requests
+        found = record_traffic(args.record_traffic, args.config, req,
+                               f"ncu log {os.path.basename(args.record_traffic)}")
+        print(json.dumps({k: len(v[1]) for k, v in found.items()}))
+        return
     if args.impl == "reference":
         run_reference(args)
         return
@@ -319,13 +386,14 @@ def main():
     dom = max(prof, key=lambda k: prof[k][0])
     dom_ms = prof[dom][0] / max(1, prof[dom][1])
     achieved_gbs = algo_bytes[dom] / (dom_ms / 1e3) / 1e9
-    traffic = kernel_traffic(dom)
+    traffic = kernel_traffic(dom, args.config, wl.requests)
     hbm_part = {"achieved": achieved_gbs, "peak": hbm, "unit": "GB/s", "frac": achieved_gbs / hbm,
                 "algorithmic_bytes_per_launch": algo_bytes[dom]}
-    if dom.startswith("window"):
-        # a dense contraction: one pass of 2 Hq W N d flops per launch, against
-        # the sustained bf16 peak (the kernel is timed inside a long step)
-        flops = 2 * wl.requests * wl.layers * wl.q_heads * wl.window * wl.seq_len * wl.head_dim
+    # one pass of the window contraction: 2 Hq W N d flops per launch
+    flops = 2 * wl.requests * wl.layers * wl.q_heads * wl.window * wl.seq_len * wl.head_dim
+    if dom.startswith("window") and flops / algo_bytes[dom] > tflops_sus * 1e3 / hbm:
+        # a dense contraction above the ridge point: against the sustained
+        # bf16 peak (the kernel is timed inside a long step)
         tf = flops / (dom_ms / 1e3) / 1e12
         roofline = {"bound": "tensor", "kernel": dom, "achieved": tf, "peak": tflops_sus,
                     "unit": "TFLOP/s", "frac": tf / tflops_sus,
