@@ -262,7 +262,8 @@ def run_reference(args):
         oracle.compress(qb, kb, vb, budget, p, threads=threads, units=units)
     secs = time.perf_counter() - t0
     value = len(units) * args.steps / secs
-    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": 0, "steps": args.steps,
+    # n_gpus echoes the launch; the work runs on rank 0's host cores only
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "impl": "reference",
