@@ -178,35 +178,41 @@ bacon_status check_seq(const bacon_ctx* c, int N, int budget)
     return BACON_OK;
 }
 
-// Encode the TMA descriptors of `pairs` (request, layer) pairs and copy them
-// to `d_maps` on the stream (K maps at [0, stride), query maps at [stride,
-// 2 stride)); skipped when the pointers and N are those of the last upload.
+// Encode the TMA descriptors of the (request, layer) pairs in slots
+// [map0, map0 + pairs) and copy them to `d_maps` on the stream (K maps at
+// [0, stride), query maps at [stride, 2 stride)); skipped when those slots
+// already hold the same pointers for this N.
 bacon_status upload_maps(const bacon_ctx* c, CUtensorMap* d_maps, CUtensorMap* h_maps,
                          cudaEvent_t ev, std::vector<const void*>& key, int& key_N, int stride,
-                         int pairs, const void* const* q, const void* const* k, int N,
+                         int map0, int pairs, const void* const* q, const void* const* k, int N,
                          cudaStream_t st)
 {
-    bool same = key_N == N && (int)key.size() == 2 * pairs;
-    for (int i = 0; same && i < pairs; ++i) same = key[2 * i] == k[i] && key[2 * i + 1] == q[i];
+    if (key_N != N || (int)key.size() != 2 * stride) {
+        key.assign(2 * stride, nullptr);  // every slot must be encoded again
+        key_N = N;
+    }
+    bool same = true;
+    for (int i = 0; same && i < pairs; ++i)
+        same = key[2 * (map0 + i)] == k[i] && key[2 * (map0 + i) + 1] == q[i];
     if (same) return BACON_OK;
     BACON_CUDA(cudaEventSynchronize(ev), "descriptor staging wait");
     for (int i = 0; i < pairs; ++i) {
-        if (!encode_rows_map(h_maps + i, k[i], c->d, (long long)c->hkv * N, kTcKBoxRows) ||
-            !encode_rows_map(h_maps + stride + i, q[i], c->d, (long long)c->hq * c->W, kTcQBoxRows))
-            return fail(BACON_ECUDA, "cuTensorMapEncodeTiled failed for pair %d", i);
+        if (!encode_rows_map(h_maps + map0 + i, k[i], c->d, (long long)c->hkv * N, kTcKBoxRows) ||
+            !encode_rows_map(h_maps + stride + map0 + i, q[i], c->d, (long long)c->hq * c->W,
+                             kTcQBoxRows))
+            return fail(BACON_ECUDA, "cuTensorMapEncodeTiled failed for pair %d", map0 + i);
     }
-    BACON_CUDA(cudaMemcpyAsync(d_maps, h_maps, sizeof(CUtensorMap) * pairs, cudaMemcpyHostToDevice, st),
-               "descriptor upload");
-    BACON_CUDA(cudaMemcpyAsync(d_maps + stride, h_maps + stride, sizeof(CUtensorMap) * pairs,
+    BACON_CUDA(cudaMemcpyAsync(d_maps + map0, h_maps + map0, sizeof(CUtensorMap) * pairs,
                                cudaMemcpyHostToDevice, st),
                "descriptor upload");
+    BACON_CUDA(cudaMemcpyAsync(d_maps + stride + map0, h_maps + stride + map0,
+                               sizeof(CUtensorMap) * pairs, cudaMemcpyHostToDevice, st),
+               "descriptor upload");
     BACON_CUDA(cudaEventRecord(ev, st), "descriptor event");
-    key.assign(2 * pairs, nullptr);
     for (int i = 0; i < pairs; ++i) {
-        key[2 * i] = k[i];
-        key[2 * i + 1] = q[i];
+        key[2 * (map0 + i)] = k[i];
+        key[2 * (map0 + i) + 1] = q[i];
     }
-    key_N = N;
     return BACON_OK;
 }
 
@@ -303,16 +309,16 @@ struct StageEvents {
 // rows' normalisers come from the caller and pass 1 is skipped.
 bacon_status window_passes(bacon_ctx* c, const Shape& s, const void* const* q,
                            const void* const* k, size_t unit0, const float* const* prefill_lse,
-                           StageEvents& prof, cudaStream_t st)
+                           StageEvents& prof, cudaStream_t st, int map0 = 0)
 {
     const int pairs = s.units / s.hkv, N = s.N;
     const int chunks = (N + kTcChunkTokens - 1) / kTcChunkTokens;
     float* lse2 = c->lse2 + unit0 * c->rows;
     float2* partial = c->partial + unit0 * chunks * c->rows;
     bacon_status rc = upload_maps(c, c->d_maps, c->h_maps, c->maps_ev, c->map_key, c->map_key_N,
-                                  kMaxPairs, pairs, q, k, N, st);
+                                  kMaxPairs, map0, pairs, q, k, N, st);
     if (rc != BACON_OK) return rc;
-    const TcArgs ta = tc_args(s, c->d_maps, c->d_maps + kMaxPairs, partial, lse2,
+    const TcArgs ta = tc_args(s, c->d_maps + map0, c->d_maps + kMaxPairs + map0, partial, lse2,
                               c->B + unit0 * N, c->Q + unit0 * N, c->E + unit0 * N, c->err);
     prof.mark(0);
     if (!prefill_lse && window_onepass_fits(s)) {
@@ -354,7 +360,7 @@ bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const vo
                              void* const* ko, void* const* vo, int32_t* const* idx,
                              cudaStream_t st, bool adaptive = false, int guaranteed = 0,
                              int32_t* counts = nullptr, size_t unit0 = 0,
-                             const float* const* prefill_lse = nullptr)
+                             const float* const* prefill_lse = nullptr, int map0 = 0)
 {
     const int pairs = R * c->layers;
     const Shape s = shape_of(c, c->layers, R, N);
@@ -378,7 +384,7 @@ bacon_status compress_device(bacon_ctx* c, int R, const void* const* q, const vo
         a.calib_budget[i] = budget;
     }
     StageEvents prof(c, st);
-    bacon_status rc = window_passes(c, s, q, k, unit0, prefill_lse, prof, st);
+    bacon_status rc = window_passes(c, s, q, k, unit0, prefill_lse, prof, st, map0);
     if (rc != BACON_OK) return rc;
 
     a.B = B;
@@ -697,7 +703,7 @@ bacon_status bacon_score_layer(bacon_ctx* ctx, bacon_state* st, int layer, const
 
     const Shape s = shape_of(ctx, 1, 1, seq_len);
     float* Eslot = st->Ering + (size_t)(layer % st->ring) * ctx->hkv * seq_len;
-    rc = upload_maps(ctx, st->d_maps, st->h_maps, st->maps_ev, st->map_key, st->map_key_N, 1, 1,
+    rc = upload_maps(ctx, st->d_maps, st->h_maps, st->maps_ev, st->map_key, st->map_key_N, 1, 0, 1,
                      &q_win, &k, seq_len, cs);
     if (rc != BACON_OK) return rc;
     const TcArgs ta = tc_args(s, st->d_maps, st->d_maps + 1, st->partial, st->lse2, st->B, st->Q,
@@ -999,6 +1005,28 @@ bacon_status bacon_compress_host(bacon_ctx* ctx, int requests, const void* q_win
     const char* qh = static_cast<const char*>(q_win);
     const char* kh = static_cast<const char*>(k);
     const char* vh = static_cast<const char*>(v);
+    const void* qs[kMaxPairs];
+    const void* ks[kMaxPairs];
+    const void* vs[kMaxPairs];
+    void* kos[kMaxPairs];
+    void* vos[kMaxPairs];
+    for (int i = 0; i < pairs; ++i) {
+        qs[i] = static_cast<const uint16_t*>(ctx->hq_buf) + q_pair * i;
+        ks[i] = static_cast<const uint16_t*>(ctx->hk_buf) + kv_pair * i;
+        vs[i] = static_cast<const uint16_t*>(v_dev ? v_dev : ctx->hv_buf) + kv_pair * i;
+        kos[i] = static_cast<uint16_t*>(ctx->hko_buf) + o_pair * i;
+        vos[i] = static_cast<uint16_t*>(ctx->hvo_buf) + o_pair * i;
+    }
+    // The TMA descriptors of every request's staging buffers go to the
+    // device first (cached across calls while the buffers stay the same): a
+    // descriptor copy queued on the compute stream after the uploads would
+    // wait behind all of them in the copy engine and hold back the first
+    // request's kernels until the last upload had landed.
+    {
+        rc = upload_maps(ctx, ctx->d_maps, ctx->h_maps, ctx->maps_ev, ctx->map_key, ctx->map_key_N,
+                         kMaxPairs, 0, pairs, qs, ks, seq_len, cs);
+        if (rc != BACON_OK) return rc;
+    }
     BACON_CUDA(cudaEventRecord(ctx->ev_done[0], cs), "event");  // uploads start after earlier work
     BACON_CUDA(cudaStreamWaitEvent(ctx->h2d, ctx->ev_done[0], 0), "event wait");
     for (int r = 0; r < requests; ++r) {
@@ -1013,18 +1041,6 @@ bacon_status bacon_compress_host(bacon_ctx* ctx, int requests, const void* q_win
         BACON_CUDA(cudaEventRecord(ctx->ev_in[r], ctx->h2d), "event");
     }
 
-    const void* qs[kMaxPairs];
-    const void* ks[kMaxPairs];
-    const void* vs[kMaxPairs];
-    void* kos[kMaxPairs];
-    void* vos[kMaxPairs];
-    for (int i = 0; i < pairs; ++i) {
-        qs[i] = static_cast<const uint16_t*>(ctx->hq_buf) + q_pair * i;
-        ks[i] = static_cast<const uint16_t*>(ctx->hk_buf) + kv_pair * i;
-        vs[i] = static_cast<const uint16_t*>(v_dev ? v_dev : ctx->hv_buf) + kv_pair * i;
-        kos[i] = static_cast<uint16_t*>(ctx->hko_buf) + o_pair * i;
-        vos[i] = static_cast<uint16_t*>(ctx->hvo_buf) + o_pair * i;
-    }
     std::vector<int> budgets(L, budget);
     int32_t* idx_pairs[kMaxPairs];
     for (int i = 0; i < pairs; ++i) idx_pairs[i] = ctx->hidx_buf + (size_t)i * ctx->hkv * kept;
@@ -1032,7 +1048,7 @@ bacon_status bacon_compress_host(bacon_ctx* ctx, int requests, const void* q_win
         BACON_CUDA(cudaStreamWaitEvent(cs, ctx->ev_in[r], 0), "event wait");
         rc = compress_device(ctx, 1, qs + r * L, ks + r * L, vs + r * L, seq_len, budgets.data(),
                              kos + r * L, vos + r * L, idx_pairs + r * L, cs, false, 0, nullptr,
-                             (size_t)r * L * ctx->hkv);
+                             (size_t)r * L * ctx->hkv, nullptr, r * L);
         if (rc != BACON_OK) return rc;
         BACON_CUDA(cudaEventRecord(ctx->ev_done[r], cs), "event");
         BACON_CUDA(cudaStreamWaitEvent(ctx->d2h, ctx->ev_done[r], 0), "event wait");
