@@ -42,7 +42,8 @@ constexpr int kSelHist = kSelBins + 64 + kSelCap;
 // kSelBins bins of 2^shift keys (plain shared-memory adds: the bins follow
 // the data's own range, so few keys share one), takes the bin where the
 // count from the top reaches k, and narrows the range to it, until a bin is
-// one key.  At most three passes for 32-bit keys.  Every thread returns the
+// one key, or until it holds at most 32 keys, which one warp then sorts.
+// At most three passes for 32-bit keys.  Every thread returns the
 // same result; blockDim.x must be a power of two from 64 to 1024.
 // kmin / kmax: this thread's share of the key range (the callers that know
 // it from an earlier pass over the keys pass it in; see radix_select_by).
@@ -164,6 +165,55 @@ __device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist
         width = (uint64_t)1 << shift;
         __syncthreads();
         if (shift == 0) return {lo, remaining, in_bin};
+        if (in_bin <= 32) {
+            // few keys left in the range: gather them (the bins are free
+            // now) and let one warp sort them instead of more passes
+            int* few = hist;
+            if (threadIdx.x == 0) *bufcnt = 0;
+            __syncthreads();
+            if (nbuf >= 0) {
+                for (int i = threadIdx.x; i < nbuf; i += blockDim.x) {
+                    const uint32_t key = buf[i];
+                    if (key >= lo && (uint64_t)(key - lo) < width) few[atomicAdd(bufcnt, 1)] = (int)key;
+                }
+            } else {
+                for (int i = threadIdx.x; i < n; i += blockDim.x) {
+                    uint32_t key = 0u;
+                    if (key_of(i, key) && key >= lo && (uint64_t)(key - lo) < width)
+                        few[atomicAdd(bufcnt, 1)] = (int)key;
+                }
+            }
+            __syncthreads();
+            if (warp == 0) {
+                // (valid, key) pairs sorted descending by a bitonic network
+                // across the lanes; invalid lanes sink to the end
+                unsigned long long v =
+                    lane < in_bin ? ((1ull << 32) | (uint32_t)few[lane]) : 0ull;
+#pragma unroll
+                for (int k = 2; k <= 32; k <<= 1) {
+#pragma unroll
+                    for (int j = k >> 1; j > 0; j >>= 1) {
+                        const unsigned long long o = __shfl_xor_sync(0xffffffffu, v, j);
+                        const bool keep_max = ((lane & k) == 0) == ((lane & j) == 0);
+                        v = keep_max ? (v > o ? v : o) : (v < o ? v : o);
+                    }
+                }
+                const uint32_t tau = (uint32_t)__shfl_sync(0xffffffffu, v, remaining - 1);
+                const bool valid = (v >> 32) != 0ull;
+                const uint32_t key = (uint32_t)v;
+                const int eq = __popc(__ballot_sync(0xffffffffu, valid && key == tau));
+                const int gt = __popc(__ballot_sync(0xffffffffu, valid && key > tau));
+                if (lane == 0) {
+                    bcast[0] = (int)tau;
+                    bcast[1] = remaining - gt;
+                    bcast[4] = eq;
+                }
+            }
+            __syncthreads();
+            const SelectResult r = {(uint32_t)bcast[0], bcast[1], bcast[4]};
+            __syncthreads();
+            return r;
+        }
         shift = shift > kSelBits ? shift - kSelBits : 0;
     }
 }
