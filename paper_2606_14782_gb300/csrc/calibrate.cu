@@ -288,17 +288,31 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
             radix_select_range(n_cand, keep, FloatKeys{Sb}, hist, bcast, skmin, skmax);
         const Segment sg = warp_segment(n_cand);
         const int eqb = eq_before_segment(Sb, sg, sel, warp_sums, &total_s);
-        int mine = 0;
-        walk_topk(Sb, sg, sel, eqb, [&](int, bool, bool in) { mine += in; });
-        const int base = warp_exclusive_scan(warp_sum(mine), warp_sums, &total_s);
         const int lane = threadIdx.x & 31;
         const uint32_t lt = (1u << lane) - 1u;
-        int pos = base;
-        walk_topk(Sb, sg, sel, eqb, [&](int i, bool, bool in) {
-            const uint32_t ball = __ballot_sync(0xffffffffu, in);
-            if (in) out[pos + __popc(ball & lt)] = i;
-            pos += __popc(ball);
-        });
+        if constexpr (PER <= 16) {
+            // membership ballots kept in registers for the emitting pass (a
+            // warp segment is at most PER x 32 candidates: N <= PER blockDim)
+            uint32_t masks[PER];
+            const int mine = walk_topk_masks_by<PER>(sg, sel, eqb, FloatKeys{Sb}, masks);
+            int pos = warp_exclusive_scan(mine, warp_sums, &total_s);
+#pragma unroll
+            for (int st = 0; st < PER; ++st) {
+                const uint32_t m = masks[st];
+                if ((m >> lane) & 1u) out[pos + __popc(m & lt)] = sg.lo + 32 * st + lane;
+                pos += __popc(m);
+            }
+        } else {
+            // longest prompts: no registers to spare, the keys are walked twice
+            int mine = 0;
+            walk_topk(Sb, sg, sel, eqb, [&](int, bool, bool in) { mine += in; });
+            int pos = warp_exclusive_scan(warp_sum(mine), warp_sums, &total_s);
+            walk_topk(Sb, sg, sel, eqb, [&](int i, bool, bool in) {
+                const uint32_t ball = __ballot_sync(0xffffffffu, in);
+                if (in) out[pos + __popc(ball & lt)] = i;
+                pos += __popc(ball);
+            });
+        }
         if (threadIdx.x == 0 && total_s != keep && a.err) atomicExch(a.err, 2);
     }
     for (int w = threadIdx.x; w < win; w += blockDim.x) out[keep + w] = N - W + w;

@@ -316,6 +316,39 @@ __device__ __forceinline__ void walk_topk_by(Segment sg, SelectResult sel, int e
     }
 }
 
+// walk_topk_by over this warp's segment that keeps each 32-element step's
+// membership ballot in masks[0, MAXSTEPS) (0 past the segment's end) and
+// returns the segment's member count, so that a later pass can emit the
+// members without reading the keys again.  MAXSTEPS must cover the segment
+// (its length / 32).
+template <int MAXSTEPS, typename KeyFn>
+__device__ __forceinline__ int walk_topk_masks_by(Segment sg, SelectResult sel, int eq_before,
+                                                  KeyFn key_of, uint32_t* masks)
+{
+    const int lane = threadIdx.x & 31;
+    const uint32_t lt = (1u << lane) - 1u;
+    int running = eq_before, total = 0;
+#pragma unroll
+    for (int st = 0; st < MAXSTEPS; ++st) {
+        const int base = sg.lo + 32 * st;
+        uint32_t m = 0u;
+        if (base < sg.hi) {
+            const int i = base + lane;
+            uint32_t key = 0u;
+            const bool valid = i < sg.hi && key_of(i, key);
+            const bool eq = valid && key == sel.tau;
+            const uint32_t ball = __ballot_sync(0xffffffffu, eq);
+            const int rank = running + __popc(ball & lt);
+            const bool in = valid && (key > sel.tau || (eq && rank < sel.need));
+            running += __popc(ball);
+            m = __ballot_sync(0xffffffffu, in);
+        }
+        masks[st] = m;
+        total += __popc(m);
+    }
+    return total;
+}
+
 // Plain float arrays (every element included).
 struct FloatKeys {
     const float* v;
