@@ -100,7 +100,10 @@ void bacon_default_params(bacon_params* p);
  * window W; odd max-pool width `pool` (1 = no pooling); default budget.
  * p may be NULL for the defaults.  Allocates the device scratch for
  * max_requests x layers x kv_heads x max_seq_len scores on the current
- * device. */
+ * device.  For tests of failure detection only: when the environment
+ * variable BACON_FAULT is "missing_arrival" at this call, the context's
+ * next two-pass window step withholds one K-tile load, its bounded pipeline
+ * waits run out and bacon_sync reports BACON_ETIMEOUT (nothing faults). */
 bacon_status bacon_init(bacon_ctx** out, int layers, int kv_heads, int q_heads,
                         int head_dim, int window, int pool, int budget,
                         const bacon_params* p);

@@ -101,7 +101,7 @@ adaptive_select_kernel(Shape s, int keep_window, AdaptArgs a)
         off += count + win;
         __syncthreads();
     }
-    if (threadIdx.x == 0 && off != H * kept_total && a.err) atomicExch(a.err, 2);
+    if (threadIdx.x == 0 && off != H * kept_total && a.err) atomicCAS(a.err, 0, 2);
 }
 
 // Flat per-layer gather: output row j of a pair belongs to the head whose
@@ -123,7 +123,7 @@ gather_flat_kernel(GatherTable tab, Shape s, const int32_t* __restrict__ counts,
     }
     const int src = tab.idx[pair][j];
     if (src < 0 || src >= s.N) {
-        if (err) atomicExch(err, 1);
+        if (err) atomicCAS(err, 0, 1);
         return;
     }
     const size_t in_off = ((size_t)h * s.N + src) * s.d;

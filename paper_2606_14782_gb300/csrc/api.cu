@@ -2,6 +2,7 @@
 // and the launch sequence of the compression step.
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cmath>
 #include <cstring>
 #include <new>
@@ -110,6 +111,10 @@ struct bacon_ctx {
     std::vector<cudaEvent_t> ev_in, ev_done;
     // per-kernel timing (bacon_profile_enable)
     int prof_on = 0;
+    // test-only fault injection, read from the environment at bacon_init
+    // (BACON_FAULT=missing_arrival): the next two-pass window step runs pass
+    // 1 with one K-tile load withheld, so its bounded waits run out
+    int fault_pending = 0;
     std::vector<cudaEvent_t> ev_free;
     std::vector<std::vector<cudaEvent_t>> ev_pending;  // 6 events per call
     std::vector<uint32_t> ev_skipped;                  // per call: stages that launched nothing
@@ -318,8 +323,8 @@ bacon_status window_passes(bacon_ctx* c, const Shape& s, const void* const* q,
     bacon_status rc = upload_maps(c, c->d_maps, c->h_maps, c->maps_ev, c->map_key, c->map_key_N,
                                   kMaxPairs, map0, pairs, q, k, N, st);
     if (rc != BACON_OK) return rc;
-    const TcArgs ta = tc_args(s, c->d_maps + map0, c->d_maps + kMaxPairs + map0, partial, lse2,
-                              c->B + unit0 * N, c->Q + unit0 * N, c->E + unit0 * N, c->err);
+    TcArgs ta = tc_args(s, c->d_maps + map0, c->d_maps + kMaxPairs + map0, partial, lse2,
+                        c->B + unit0 * N, c->Q + unit0 * N, c->E + unit0 * N, c->err);
     prof.mark(0);
     if (!prefill_lse && window_onepass_fits(s)) {
         // the unit's logits stay in tensor memory: one kernel, one pass over K
@@ -339,7 +344,14 @@ bacon_status window_passes(bacon_ctx* c, const Shape& s, const void* const* q,
         for (int i = 0; i < pairs; ++i) t.lse[i] = prefill_lse[i];
         BACON_CUDA(launch_lse_from_prefill(s, t, lse2, st), "normaliser conversion launch");
     } else {
-        BACON_CUDA(launch_window_stats_tc(ta, st), "window_stats launch");
+        if (c->fault_pending) {
+            TcArgs tf = ta;
+            tf.fault = 1;
+            c->fault_pending = 0;
+            BACON_CUDA(launch_window_stats_tc(tf, st), "window_stats launch");
+        } else {
+            BACON_CUDA(launch_window_stats_tc(ta, st), "window_stats launch");
+        }
         prof.mark(1);
         BACON_CUDA(launch_window_combine(s, ta.chunks, partial, lse2, st), "window_combine launch");
     }
@@ -618,6 +630,8 @@ bacon_status bacon_init(bacon_ctx** out, int layers, int kv_heads, int q_heads, 
         delete c;
         return fail(BACON_ENOMEM, "device allocation failed: %s", cudaGetErrorString(e));
     }
+    const char* fault = std::getenv("BACON_FAULT");  // tests only
+    if (fault && std::strcmp(fault, "missing_arrival") == 0) c->fault_pending = 1;
     *out = c;
     return BACON_OK;
 }

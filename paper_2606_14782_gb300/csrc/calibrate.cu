@@ -313,7 +313,7 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
                 pos += __popc(ball);
             });
         }
-        if (threadIdx.x == 0 && total_s != keep && a.err) atomicExch(a.err, 2);
+        if (threadIdx.x == 0 && total_s != keep && a.err) atomicCAS(a.err, 0, 2);
     }
     for (int w = threadIdx.x; w < win; w += blockDim.x) out[keep + w] = N - W + w;
 }

@@ -20,7 +20,7 @@ gather_kernel(GatherTable tab, Shape s, int* __restrict__ err)
     if (j >= kept) return;
     const int src = tab.idx[pair][(size_t)h * kept + j];
     if (src < 0 || src >= s.N) {
-        if (err) atomicExch(err, 1);
+        if (err) atomicCAS(err, 0, 1);
         return;
     }
     const size_t in_off = ((size_t)h * s.N + src) * s.d;

@@ -84,7 +84,7 @@ struct Bars {
 __device__ inline void raise_abort(const Bars& b, int* err)
 {
     tc::st_shared_volatile(b.abort(), 1u);
-    if (err) atomicExch(err, tc::kErrTimeout);
+    if (err) atomicCAS(err, 0, tc::kErrTimeout);
 }
 
 __device__ inline void unit_range(int units, int* u0, int* u1)

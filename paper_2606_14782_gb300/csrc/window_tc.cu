@@ -138,7 +138,7 @@ __device__ inline Bars bars_at(uint8_t* p, int stages)
 __device__ inline void raise_abort(const Bars& b, int* err)
 {
     tc::st_shared_volatile(b.abort(), 1u);
-    if (err) atomicExch(err, tc::kErrTimeout);
+    if (err) atomicCAS(err, 0, tc::kErrTimeout);
 }
 
 // Range of global chunks [c0, c1) owned by this CTA.
@@ -253,6 +253,9 @@ __device__ __forceinline__ void produce(const TcArgs& a, const Smem& L, uint8_t*
             for (int t = ci * kTilesPerChunk; t < t1; ++t, ++kt) {
                 const int st = kt % stages, n = kt / stages;
                 if (!tc::mbar_wait(b.k_empty(st), (n & 1) ^ 1, b.abort())) { ok = false; break; }
+                // injected fault (tests only): the first load never arrives, so
+                // the MMA thread's bounded wait runs out and the CTA aborts
+                if (PASS == 1 && a.fault == 1 && blockIdx.x == 0 && kt == 0) continue;
                 tc::mbar_arrive_expect_tx(b.k_full(st), L.k_stage);
                 for (int kh = 0; kh < H; ++kh)
                     tc::tma_load_2d_hint(sm + L.k + st * L.k_stage + kh * kTileTok * 128,

@@ -21,6 +21,8 @@ struct TcArgs {
     float* Q;
     float* E;
     int* err;                  // device error word (timeouts)
+    int fault = 0;             // test-only fault injection: 1 = CTA 0 of pass 1 never
+                               // issues its first K-tile load (a missing arrival)
 };
 
 constexpr int kTcChunkTokens = 1024;
