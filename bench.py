@@ -152,7 +152,11 @@ KERNEL_SOURCES = [
 ]
 
 
-def record_traffic(csv_path: str, workload: str, requests: int, command: str):
+TRAFFIC_PATH = os.path.join(ROOT, "profiles", "traffic.json")
+
+
+def record_traffic(csv_path: str, workload: str, requests: int, command: str,
+                   path: str = TRAFFIC_PATH):
     """Average dram__bytes_read.sum + dram__bytes_write.sum per launch of each
     library kernel in an ncu --csv log, per request, into traffic.json."""
     import csv
@@ -169,7 +173,6 @@ def record_traffic(csv_path: str, workload: str, requests: int, command: str):
         scale = {"byte": 1, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9}[unit]
         key = (r[col["ID"]], r[col["Kernel Name"]])
         per_launch[key] = per_launch.get(key, 0.0) + float(r[col["Metric Value"]].replace(",", "")) * scale
-    path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
             rec = json.load(f)
@@ -195,12 +198,11 @@ def record_traffic(csv_path: str, workload: str, requests: int, command: str):
     return found
 
 
-def kernel_traffic(kernel: str, workload: str, requests: int):
+def kernel_traffic(kernel: str, workload: str, requests: int, path: str = TRAFFIC_PATH):
     """DRAM bytes per launch from the committed ncu summary of this kernel on
     this workload (scaled to `requests`: traffic grows with the units), or
     None when there is none or the kernel's sources changed since the
     counters were taken."""
-    path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
             rec = json.load(f)[workload][kernel]

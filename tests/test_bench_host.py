@@ -1,0 +1,90 @@
+"""Host-side logic of bench.py, on the CPU: the traffic record written from an
+ncu log and read back (per workload, scaled by the requests of a launch,
+voided when the kernel's sources change), and the reference arm's JSON line."""
+
+import json
+import os
+import subprocess
+import sys
+
+import pytest
+
+import bench
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+HEADER = ('"ID","Process ID","Process Name","Host Name","Kernel Name","Context","Stream",'
+          '"Block Size","Grid Size","Device","CC","Section Name","Metric Name","Metric Unit",'
+          '"Metric Value"\n')
+
+
+def _row(i, kernel, metric, unit, value):
+    return (f'"{i}","1","python3","h","{kernel}","1","7","(576, 1, 1)","(152, 1, 1)","0","10.3",'
+            f'"Command line profiler metrics","{metric}","{unit}","{value}"\n')
+
+
+def _ncu_log(tmp_path):
+    k1 = "void unnamed>::window_tc_kernel<128, 1>(TcArgs, unnamed>::Plan)"
+    k2 = "void unnamed>::window_tc_kernel<128, 2>(TcArgs, unnamed>::Plan)"
+    cal = "void unnamed>::calibrate_select_kernel<1024, 16>(Shape, Calib, CalibArgs)"
+    text = ("==PROF== Connected to process 1\n" + HEADER
+            + _row(0, k1, "dram__bytes_read.sum", "Mbyte", "480.5")
+            + _row(0, k1, "dram__bytes_write.sum", "byte", "500000")
+            + _row(0, k1, "gpu__time_duration.sum", "us", "197.0")
+            + _row(1, k2, "dram__bytes_read.sum", "Gbyte", "0.48")
+            + _row(1, k2, "dram__bytes_write.sum", "Kbyte", "1,625.3")
+            + _row(2, cal, "dram__bytes_read.sum", "byte", "14790912")
+            + _row(2, cal, "dram__bytes_write.sum", "byte", "0")
+            + _row(3, cal, "dram__bytes_read.sum", "byte", "14790000")
+            + _row(3, cal, "dram__bytes_write.sum", "byte", "0"))
+    p = tmp_path / "log.csv"
+    p.write_text(text)
+    return str(p)
+
+
+def test_record_and_read_traffic(tmp_path):
+    out = str(tmp_path / "traffic.json")
+    found = bench.record_traffic(_ncu_log(tmp_path), "gui", 1, "ncu ...", path=out)
+    assert set(found) == {"window_stats", "window_scores", "calibrate_select"}
+    rec = json.load(open(out))["gui"]
+    assert rec["window_stats"]["dram_bytes_per_request"] == pytest.approx(480.5e6 + 5e5)
+    assert rec["window_scores"]["dram_bytes_per_request"] == pytest.approx(0.48e9 + 1625.3e3)
+    # two launches of the calibration kernel: their mean
+    assert rec["calibrate_select"]["launches"] == 2
+    assert rec["calibrate_select"]["dram_bytes_per_request"] == pytest.approx(14790456.0)
+    # read back for a 4-request launch of the same workload
+    assert bench.kernel_traffic("window_stats", "gui", 4, path=out) == pytest.approx(4 * (480.5e6 + 5e5))
+    # another workload, or a kernel without a record: nothing
+    assert bench.kernel_traffic("window_stats", "llava", 1, path=out) is None
+    assert bench.kernel_traffic("gather", "gui", 1, path=out) is None
+    # a record whose sources changed since the capture is void
+    rec_all = json.load(open(out))
+    rec_all["gui"]["window_stats"]["code_sha256_16"] = "0" * 16
+    json.dump(rec_all, open(out, "w"))
+    assert bench.kernel_traffic("window_stats", "gui", 4, path=out) is None
+    assert bench.kernel_traffic("window_scores", "gui", 4, path=out) is not None
+
+
+def test_source_digest_ignores_comments():
+    # the digest of the committed sources is stable and comment-insensitive by construction
+    d = bench.source_digest(["gather.cu", "common.cuh"])
+    assert len(d) == 16 and d == bench.source_digest(["gather.cu", "common.cuh"])
+    assert d != bench.source_digest(["gather.cu"])
+
+
+def test_reference_arm_json_line():
+    proc = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+                           "--config", "tiny", "--steps", "1", "--warmup", "0"],
+                          capture_output=True, text=True, timeout=600, cwd=ROOT)
+    assert proc.returncode == 0, proc.stderr[-2000:]
+    line = json.loads(proc.stdout.strip().splitlines()[-1])
+    for key in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+                "higher_is_better", "scaling", "vs_baseline", "dtype", "data", "config",
+                "cpu_baseline", "e2e"):
+        assert key in line, key
+    assert line["impl"] == "reference"
+    assert line["value"] > 0 and line["higher_is_better"] is True
+    assert line["e2e"]["value"] == line["value"]
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
+    assert line["config"]["workload"].startswith("tiny")
