@@ -9,6 +9,8 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "bacon.h"
 #include "common.cuh"
 #include "window_tc.h"
@@ -289,9 +291,19 @@ struct StageEvents {
         }
     }
     uint32_t skipped = 0;
+    bool range_open = false;
+    // stage boundary i: CUDA-event timing (bacon_profile_enable) and an NVTX
+    // range per stage ("bacon/window_stats", ...) around its launches, for
+    // profilers (no cost without one attached)
     void mark(int i)
     {
         if (c->prof_on && ev[i]) cudaEventRecord(ev[i], st);
+        static const char* const names[BACON_PROFILE_STAGES] = {
+            "bacon/window_stats", "bacon/window_combine", "bacon/window_scores",
+            "bacon/calibrate_select", "bacon/gather"};
+        if (range_open) nvtxRangePop();
+        range_open = i < BACON_PROFILE_STAGES;
+        if (range_open) nvtxRangePushA(names[i]);
     }
     void skip(int i) { skipped |= 1u << i; }  // stage i launched nothing in this call
     void commit()
@@ -304,6 +316,7 @@ struct StageEvents {
     }
     ~StageEvents()
     {
+        if (range_open) nvtxRangePop();
         for (cudaEvent_t e : ev)  // a call that failed before commit()
             if (e) c->ev_free.push_back(e);
     }
