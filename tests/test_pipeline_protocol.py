@@ -16,7 +16,9 @@ every schedule finishes and every wait returns in its own phase.  The
 variant in which the merging group does not first wait for the slot's
 previous read (the kernels' earlier protocol) fails the check.  The one-pass
 kernel (logits resident in TMEM, two CTA-wide syncs per unit) is modelled
-the same way.
+the same way, and so is the abort path: with one K-tile load withheld (the
+failure-detection test's injected missing arrival), every role's bounded
+wait gives up, the CTA drains the copies it issued and every role finishes.
 """
 
 import random
@@ -174,12 +176,6 @@ def cta_range(units, chunks_per_unit, total_ctas, cta):
     return [(g // chunks_per_unit, g % chunks_per_unit) for g in range(c0, c1)]
 
 
-def cta_range(units, chunks_per_unit, total_ctas, cta):
-    total = units * chunks_per_unit
-    c0, c1 = cta * total // total_ctas, (cta + 1) * total // total_ctas
-    return [(g // chunks_per_unit, g % chunks_per_unit) for g in range(c0, c1)]
-
-
 def _cases(n=40, seed=3):
     rng = random.Random(seed)
     out = []
@@ -312,4 +308,189 @@ def simulate_onepass(n_units, ntiles, stages, epi_warps, seed):
 def test_onepass_protocol(n_units, ntiles, stages):
     for seed in range(6):
         fault = simulate_onepass(n_units, ntiles, stages, 8, seed)
+        assert fault is None, (seed, fault)
+
+
+# ------------------------------------------------ abort path (missing arrival)
+
+def simulate_abort(chunks, n_tiles, tpc, jobs_per_tile, nbuf, stages, q_slots, pass2, seed,
+                   limit=400):
+    """The two-pass kernel with the first K-tile load withheld.  Waits are
+    bounded (`limit` polls stand for the clock limit) and also give up once
+    the CTA's abort flag is set, except the drains, which only have the
+    clock; a role whose wait gives up raises the flag and leaves its loops,
+    as the kernels do.  Returns None when every role finishes with no copy
+    still in flight, else what went wrong."""
+    rnd = random.Random(seed)
+    t_full = [Bar(1, f"t_full{i}") for i in range(nbuf)]
+    t_empty = [Bar(16, f"t_empty{i}") for i in range(nbuf)]
+    k_full = [Bar(1, f"k_full{i}") for i in range(stages)]
+    k_empty = [Bar(1, f"k_empty{i}") for i in range(stages)]
+    q_full = [Bar(2 if pass2 else 1, f"q_full{i}") for i in range(q_slots)]
+    q_empty = [Bar(1, f"q_empty{i}") for i in range(q_slots)]
+    x_full = {(p, q): Bar(3, f"x_full{p}{q}") for p in range(2) for q in range(4)}
+    x_empty = {(p, q): Bar(1, f"x_empty{p}{q}") for p in range(2) for q in range(4)}
+    drain = Bar(1, "drain")
+    tma, commits = [], []
+    abort = [False]
+    ok = {}
+
+    def bwait(bar, k, key, flag=True):
+        """Bounded wait; its outcome lands in ok[key]."""
+        polls = 0
+        while (bar.phase & 1) == (k & 1):
+            if (flag and abort[0]) or polls > limit:
+                ok[key] = False
+                return
+            polls += 1
+            yield
+        ok[key] = True
+
+    def tiles_of(ci):
+        return range(ci * tpc, min(n_tiles, (ci + 1) * tpc))
+
+    def producer():
+        cur, qloads, kt = -1, 0, 0
+        good = True
+        for u, ci in chunks:
+            if u != cur:
+                slot, use = qloads % q_slots, qloads // q_slots
+                yield from bwait(q_empty[slot], use - 1, "p")
+                if not ok["p"]:
+                    good = False
+                    break
+                tma.append(q_full[slot])
+                if pass2:
+                    yield
+                    q_full[slot].arrive()
+                qloads += 1
+                cur = u
+            for _ in tiles_of(ci):
+                st, n = kt % stages, kt // stages
+                yield from bwait(k_empty[st], n - 1, "p")
+                if not ok["p"]:
+                    good = False
+                    break
+                if kt > 0:          # the first load is withheld
+                    tma.append(k_full[st])
+                kt += 1
+                yield
+            if not good:
+                break
+        if not good:
+            abort[0] = True
+        for st in range(min(stages, kt)):
+            last = kt - 1 - ((kt - 1 - st) % stages)
+            yield from bwait(k_full[st], last // stages, "pd", flag=False)
+        for slot in range(min(q_slots, qloads)):
+            last = qloads - 1 - ((qloads - 1 - slot) % q_slots)
+            yield from bwait(q_full[slot], last // q_slots, "pd", flag=False)
+
+    def mma():
+        cur, cur_slot, qwaits, kt, job = -1, 0, 0, 0, 0
+        good = True
+        for u, ci in chunks:
+            if u != cur:
+                if cur >= 0:
+                    commits.append(q_empty[cur_slot])
+                slot, use = qwaits % q_slots, qwaits // q_slots
+                yield from bwait(q_full[slot], use, "m")
+                if not ok["m"]:
+                    good = False
+                    break
+                qwaits += 1
+                cur, cur_slot = u, slot
+            for _ in tiles_of(ci):
+                st, n = kt % stages, kt // stages
+                yield from bwait(k_full[st], n, "m")
+                if not ok["m"]:
+                    good = False
+                    break
+                if st == 0 and n == 0:
+                    raise Fault("an MMA read the K stage whose load never arrived")
+                kt += 1
+                for _ in range(jobs_per_tile):
+                    buf, nb = job % nbuf, job // nbuf
+                    job += 1
+                    yield from bwait(t_empty[buf], nb - 1, "m")
+                    if not ok["m"]:
+                        good = False
+                        break
+                    commits.append(t_full[buf])
+                    yield
+                if not good:
+                    break
+                commits.append(k_empty[st])
+            if not good:
+                break
+        if not good:
+            abort[0] = True
+        commits.append(drain)
+        yield from bwait(drain, 0, "md", flag=False)
+        if not ok["md"]:
+            raise Fault("the MMA drain did not complete")
+
+    def epilogue(q, g):
+        job = n = 0
+        key = f"e{q}{g}"
+        for u, ci in chunks:
+            ts = list(tiles_of(ci))
+            for i, _ in enumerate(ts):
+                for _ in range(jobs_per_tile):
+                    buf, nb = job % nbuf, job // nbuf
+                    job += 1
+                    yield from bwait(t_full[buf], nb, key)
+                    if not ok[key]:
+                        abort[0] = True
+                        return
+                    yield
+                    t_empty[buf].arrive()
+                if not pass2 and i != len(ts) - 1:
+                    continue
+                slots = 2 if pass2 else 1
+                par, use, merger = n % slots, n // slots, n & 3
+                n += 1
+                yield from bwait(x_empty[(par, q)], use - 1, key)
+                if not ok[key]:
+                    abort[0] = True
+                    return
+                if g != merger:
+                    yield
+                    x_full[(par, q)].arrive()
+                else:
+                    yield from bwait(x_full[(par, q)], use, key)
+                    if not ok[key]:
+                        abort[0] = True
+                        return
+                    yield
+                    x_empty[(par, q)].arrive()
+
+    procs = [producer(), mma()] + [epilogue(q, g) for q in range(4) for g in range(4)]
+    live = list(range(len(procs)))
+    for _ in range(2000000):
+        if not live:
+            if tma:
+                return "a copy was still in flight when the CTA finished"
+            return None if abort[0] else "no role noticed the missing arrival"
+        r = rnd.random()
+        if tma and r < 0.25:
+            tma.pop(rnd.randrange(len(tma))).arrive()
+            continue
+        if commits and r < 0.5:
+            commits.pop(0).arrive()
+            continue
+        i = rnd.choice(live)
+        try:
+            next(procs[i])
+        except StopIteration:
+            live.remove(i)
+        except Fault as f:
+            return str(f)
+    return "deadlock"
+
+
+@pytest.mark.parametrize("chunks,n_tiles,jobs,nbuf,stages,q_slots,pass2", _cases(12, seed=11))
+def test_missing_arrival_ends_every_role(chunks, n_tiles, jobs, nbuf, stages, q_slots, pass2):
+    for seed in range(3):
+        fault = simulate_abort(chunks, n_tiles, 8, jobs, nbuf, stages, q_slots, pass2, seed)
         assert fault is None, (seed, fault)
