@@ -48,7 +48,14 @@
  * max_requests); BACON_ENOMEM when device or host allocation fails;
  * BACON_ECUDA for a CUDA launch or copy failure; BACON_ESTATE when layers
  * of a request are scored out of order or select runs before any layer was
- * scored.  A context must not be used from two threads at once.
+ * scored; BACON_EUNSUPPORTED for sizes beyond the allocation-free entry
+ * point's static scratch.  Errors found on the device are latched in the
+ * context and returned by the next bacon_sync (the first one wins):
+ * BACON_ETIMEOUT when a kernel's bounded pipeline wait (about a second) ran
+ * out, after which the kernel drained its own work and returned, so the
+ * context stays usable; BACON_EINVAL when bacon_compact was given an index
+ * outside [0, seq_len).  A context must not be used from two threads at
+ * once.
  */
 #ifndef BACON_H
 #define BACON_H
