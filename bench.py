@@ -235,10 +235,16 @@ def cpu_baseline(wl, budget):
     units = [(r, l, h) for r in range(wl.requests) for l in range(layers)
              for h in range(wl.kv_heads)]
     secs = oracle_sample(wl, budget, units, threads)
+    # the same oracle on one host thread (layer 0 of the first two kv-heads)
+    one = units[:min(2, len(units))]
+    one_secs = oracle_sample(wl, budget, one, 1)
     return {"value": len(units) / secs, "unit": UNIT, "cores": threads, "kind": "oracle",
             "sample": f"{len(units)} layer-heads (layers 0-{layers - 1} of every request and "
                       f"kv-head) of the same workload, double precision, {threads} threads, "
-                      f"{secs:.1f} s wall"}
+                      f"{secs:.1f} s wall",
+            "single_thread": {"value": len(one) / one_secs, "unit": UNIT, "cores": 1,
+                              "sample": f"{len(one)} layer-heads, one thread, "
+                                        f"{one_secs:.2f} s wall"}}
 
 
 def run_reference(args):

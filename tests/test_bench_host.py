@@ -88,3 +88,12 @@ def test_reference_arm_json_line():
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
     assert line["config"]["workload"].startswith("tiny")
+
+
+def test_cpu_baseline_reports_threads_and_one_thread():
+    from paper_2606_14782_gb300 import workloads
+    wl = workloads.CONFIGS["tiny"]
+    cb = bench.cpu_baseline(wl, wl.budgets[0])
+    assert cb["kind"] == "oracle" and cb["unit"] == bench.UNIT and cb["value"] > 0
+    assert cb["cores"] == min(os.cpu_count() or 1, wl.requests * wl.kv_heads)
+    assert cb["single_thread"]["cores"] == 1 and cb["single_thread"]["value"] > 0
