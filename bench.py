@@ -53,6 +53,11 @@ def parse():
     return ap.parse_args()
 
 
+# exponentials per clock per SM of the special-function unit (ex2): the
+# nominal rate of this part (Blackwell Ultra doubles sm_100's 16)
+SFU_EX2_PER_CLK_PER_SM = 32
+
+
 def peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -62,6 +67,16 @@ def peaks():
                 float(p.get("bf16_tflops_sustained", p["bf16_tflops"])), "measured")
     except Exception:
         return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def max_sm_mhz() -> float:
+    """Maximum SM clock recorded beside the measured peaks (else 2070 MHz,
+    this part's maximum)."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f).get("sm_max_mhz", 2070.0))
+    except Exception:
+        return 2070.0
 
 
 def config_dict(wl, budget, n_gpus):
@@ -215,36 +230,84 @@ def kernel_traffic(kernel: str, workload: str, requests: int, path: str = TRAFFI
 
 # ---------------------------------------------------- CPU oracle legs
 
-def oracle_sample(wl, budget, units, threads):
-    """Time the CPU oracle on `units` of a same-shaped host workload."""
+def oracle_sample(qb, kb, vb, wl, budget, units, threads):
+    """Time the CPU oracle on `units` of the given bf16 inputs (bit patterns);
+    returns (seconds, the oracle's per-unit results)."""
     import oracle
-    from paper_2606_14782_gb300 import workloads
 
-    layers_needed = max(l for _, l, _ in units) + 1
-    host = workloads.generate(wl.with_(layers=layers_needed), seed=0, device="cpu")
-    qb, kb, vb = (workloads.bf16_bits(t) for t in (host.qwin, host.k, host.v))
     p = oracle.Params(pool_kernel=wl.pool)
     t0 = time.perf_counter()
-    oracle.compress(qb, kb, vb, budget, p, threads=threads, units=units)
-    return time.perf_counter() - t0
+    res = oracle.compress(qb, kb, vb, budget, p, threads=threads, units=units, keep_scores=True)
+    return time.perf_counter() - t0, res
 
 
-def cpu_baseline(wl, budget):
+def boundary_swaps(gpu_idx, orc_idx, orc_S, N, W, budget, rtol=2e-3, atol=1e-5):
+    """(swaps, allowed) for one unit: positions kept by the GPU only, and
+    whether every position kept by one side only has an oracle score within
+    atol + rtol |S| of the oracle's boundary score."""
+    import numpy as np
+    g, o = set(gpu_idx.tolist()), set(orc_idx.tolist())
+    if g == o:
+        return 0, True
+    n_cand, keep = N - W, min(budget, N) - W
+    S = np.asarray(orc_S, dtype=np.float64)
+    order = np.lexsort((np.arange(n_cand), -S[:n_cand]))
+    thr = S[order[keep - 1]]
+    band = atol + rtol * abs(thr)
+    ok = all(abs(S[i] - thr) <= band for i in g ^ o if i < n_cand)
+    return len(g - o), ok and len(g - o) == len(o - g)
+
+
+def cpu_baseline(wl, budget, host, gpu_idx):
+    """The oracle on the bench's own inputs (layers 0-1 of every request and
+    kv-head), on the host cores; its selections are compared with the GPU's
+    for those units (boundary swaps counted)."""
     threads = min(os.cpu_count() or 1, wl.requests * wl.kv_heads)
     layers = min(2, wl.layers)
     units = [(r, l, h) for r in range(wl.requests) for l in range(layers)
              for h in range(wl.kv_heads)]
-    secs = oracle_sample(wl, budget, units, threads)
+    qb, kb, vb = host
+    secs, res = oracle_sample(qb, kb, vb, wl, budget, units, threads)
+    swaps, allowed = 0, True
+    for (r, l, h), o in res.items():
+        n, ok = boundary_swaps(gpu_idx[r, l, h], o["idx"], o["S"], wl.seq_len, wl.window, budget)
+        swaps += n
+        allowed = allowed and ok
     # the same oracle on one host thread (layer 0 of the first two kv-heads)
     one = units[:min(2, len(units))]
-    one_secs = oracle_sample(wl, budget, one, 1)
+    one_secs, _ = oracle_sample(qb, kb, vb, wl, budget, one, 1)
     return {"value": len(units) / secs, "unit": UNIT, "cores": threads, "kind": "oracle",
             "sample": f"{len(units)} layer-heads (layers 0-{layers - 1} of every request and "
-                      f"kv-head) of the same workload, double precision, {threads} threads, "
+                      f"kv-head) of the timed inputs, double precision, {threads} threads, "
                       f"{secs:.1f} s wall",
             "single_thread": {"value": len(one) / one_secs, "unit": UNIT, "cores": 1,
                               "sample": f"{len(one)} layer-heads, one thread, "
-                                        f"{one_secs:.2f} s wall"}}
+                                        f"{one_secs:.2f} s wall"},
+            "sample_selection_check": {"units": len(units), "boundary_swaps": swaps,
+                                       "all_within_band": allowed}}
+
+
+SWAP_LOG_PATH = os.path.join(ROOT, "profiles", "boundary_swaps.json")
+
+
+def logged_swaps(path: str = SWAP_LOG_PATH):
+    """Per-case boundary-swap counts of the committed parity log (every unit
+    of each paper-shaped configuration against the oracle), with whether the
+    kernels changed since it was written."""
+    try:
+        with open(path) as f:
+            doc = json.load(f)
+    except (FileNotFoundError, ValueError):
+        return None
+    csrc = os.path.join(ROOT, "paper_2606_14782_gb300", "csrc")
+    names = sorted(n for n in os.listdir(csrc) if n.endswith((".cu", ".cuh", ".h")))
+    current = doc.get("code_sha256_16") == source_digest(names)
+    cases = {k: {"swaps": v["swaps"], "units": v["units_checked"],
+                 "selected_per_unit": v["selected_per_unit"],
+                 "max_gap_over_band": round(v["max_gap_over_band"], 3)}
+             for k, v in doc.get("cases", {}).items()
+             if not k.startswith(("edge ", "fuzz "))}
+    return {"source": "profiles/boundary_swaps.json", "current_code": current, "cases": cases}
 
 
 def run_reference(args):
@@ -312,6 +375,57 @@ def reduce_step_time(ms: float, world: int, device) -> float:
 def job_throughput(units_per_rank: int, world: int, ms: float) -> float:
     """Whole-job layer-heads per second: every rank's units over the slowest time."""
     return world * units_per_rank / (ms / 1e3)
+
+
+def fused_attention_lse(wl, x, dev):
+    """The window rows' natural-log softmax normalisers [R, L, Hq, W] as a
+    prefill attention kernel exports them: PyTorch's fused memory-efficient
+    attention (bf16, bottom-right causal mask as an additive bias, keys
+    repeated over each kv-head's query group) returns its log-sum-exp beside
+    the output.  Falls back to a plain fp32 computation when that kernel is
+    unavailable; returns (lse, source)."""
+    import torch
+    R, Ly, Hq, W, d = x.qwin.shape
+    N, G = wl.seq_len, wl.group
+    pos = torch.arange(N, device=dev)
+    hidden = pos[None, :] > (N - W + torch.arange(W, device=dev))[:, None]
+    out = torch.empty((R, Ly, Hq, W), dtype=torch.float32, device=dev)
+    op = getattr(torch.ops.aten, "_scaled_dot_product_efficient_attention", None)
+    try:
+        if op is None:
+            raise RuntimeError("no fused memory-efficient attention in this PyTorch")
+        bias = torch.zeros((W, N), dtype=torch.bfloat16, device=dev)
+        bias.masked_fill_(hidden, float("-inf"))
+        bias = bias.expand(1, Hq, W, N).contiguous()
+        for r in range(R):
+            for l in range(Ly):
+                k = x.k[r, l].repeat_interleave(G, dim=0).unsqueeze(0)
+                v = x.v[r, l].repeat_interleave(G, dim=0).unsqueeze(0)
+                res = op(x.qwin[r, l].unsqueeze(0), k, v, bias, True, 0.0, False, scale=d ** -0.5)
+                out[r, l] = res[1][0, :, :W].float()
+        return out, "log-sum-exp output of PyTorch's fused memory-efficient attention (bf16)"
+    except RuntimeError as e:
+        for r in range(R):
+            for l in range(Ly):
+                q = x.qwin[r, l].float().view(wl.kv_heads, G, W, d)
+                s_ = torch.einsum("hgwd,hnd->hgwn", q, x.k[r, l].float()) / d ** 0.5
+                out[r, l] = torch.logsumexp(s_.masked_fill(hidden, float("-inf")), -1).reshape(Hq, W)
+        return out, f"plain fp32 PyTorch (fused attention unavailable: {str(e)[:80]})"
+
+
+def timed(fn, steps, stream):
+    """Device time per call of fn() over `steps` calls (CUDA events on the
+    launching stream, synchronised on both sides)."""
+    import torch
+    torch.cuda.synchronize()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(steps):
+        fn()
+    b.record(stream)
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / steps
 
 
 def main():
@@ -383,11 +497,21 @@ def main():
     prof = ctx.profile_read()
     ctx.profile(False)
     ctx.sync()
-    ms = reduce_step_time(e0.elapsed_time(e1) / args.steps, world, dev)
+    region_ms = e0.elapsed_time(e1)
+    ms = reduce_step_time(region_ms / args.steps, world, dev)
 
     units = wl.requests * wl.layers * wl.kv_heads
     value = job_throughput(units, world, ms)
     hbm, tflops, tflops_sus, peak_src = peaks()
+    # a kernel timed inside a sub-second region runs at burst clocks: judge
+    # it against the burst bf16 peak; the sustained one is for a region of
+    # seconds, where the power cap pulls the clocks down
+    short = region_ms < 1000.0
+    tc_peak = tflops if short else tflops_sus
+    tc_kind = "burst" if short else "sustained"
+    sm_mhz = (clocks or {}).get("sm_mhz") or max_sm_mhz()
+    n_sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    sfu_peak = SFU_EX2_PER_CLK_PER_SM * n_sms * sm_mhz * 1e6  # exponentials per second
 
     # per-kernel times measured live (CUDA events around each launch)
     K_bytes = wl.requests * wl.layers * wl.kv_heads * wl.seq_len * wl.head_dim * 2
@@ -401,29 +525,55 @@ def main():
         "calibrate_select": tok * (4 + 4 * (1 + min(4, wl.layers - 1))) + units * kept * 4,
         "gather": 4 * units * kept * wl.head_dim * 2 + units * kept * 4,
     }
+    # one pass of the window contraction: 2 Hq W N d flops and Hq W N
+    # exponentials per launch
+    flops = 2 * wl.requests * wl.layers * wl.q_heads * wl.window * wl.seq_len * wl.head_dim
+    exps = wl.requests * wl.layers * wl.q_heads * wl.window * wl.seq_len
     total = sum(t for t, _ in prof.values())
-    kernels = {k: {"ms_per_launch": (t / n if n else None), "share": (t / total if total else None)}
-               for k, (t, n) in prof.items() if n}
+    kernels = {}
+    for k, (t, n) in prof.items():
+        if not n:
+            continue
+        kms = t / n
+        e = {"ms_per_launch": kms, "share": (t / total if total else None),
+             "algorithmic_gbs": algo_bytes[k] / (kms / 1e3) / 1e9}
+        if k in ("window_stats", "window_scores"):
+            e["tflops"] = flops / (kms / 1e3) / 1e12
+            e["sfu_ex2_frac"] = exps / (kms / 1e3) / sfu_peak
+        kernels[k] = e
     dom = max(prof, key=lambda k: prof[k][0])
     dom_ms = prof[dom][0] / max(1, prof[dom][1])
     achieved_gbs = algo_bytes[dom] / (dom_ms / 1e3) / 1e9
     traffic = kernel_traffic(dom, args.config, wl.requests)
     hbm_part = {"achieved": achieved_gbs, "peak": hbm, "unit": "GB/s", "frac": achieved_gbs / hbm,
                 "algorithmic_bytes_per_launch": algo_bytes[dom]}
-    # one pass of the window contraction: 2 Hq W N d flops per launch
-    flops = 2 * wl.requests * wl.layers * wl.q_heads * wl.window * wl.seq_len * wl.head_dim
-    if dom.startswith("window") and flops / algo_bytes[dom] > tflops_sus * 1e3 / hbm:
-        # a dense contraction above the ridge point: against the sustained
-        # bf16 peak (the kernel is timed inside a long step)
+    if dom.startswith("window") and flops / algo_bytes[dom] > tc_peak * 1e3 / hbm:
+        # a dense contraction above the ridge point: against the bf16 peak
         tf = flops / (dom_ms / 1e3) / 1e12
-        roofline = {"bound": "tensor", "kernel": dom, "achieved": tf, "peak": tflops_sus,
-                    "unit": "TFLOP/s", "frac": tf / tflops_sus,
-                    "peak_source": f"{peak_src} (bf16, sustained)", "traffic": traffic,
-                    "algorithmic_flops_per_launch": flops, "hbm": hbm_part}
+        roofline = {"bound": "tensor", "kernel": dom, "achieved": tf, "peak": tc_peak,
+                    "unit": "TFLOP/s", "frac": tf / tc_peak,
+                    "peak_source": f"{peak_src} bf16 {tc_kind} (timed region {region_ms:.0f} ms, "
+                                   f"SM clock median {sm_mhz:.0f} MHz)",
+                    "traffic": traffic, "algorithmic_flops_per_launch": flops,
+                    "sfu": {"ex2_per_launch": exps,
+                            "achieved_per_s": exps / (dom_ms / 1e3), "peak_per_s": sfu_peak,
+                            "frac": exps / (dom_ms / 1e3) / sfu_peak,
+                            "peak_source": f"nominal {SFU_EX2_PER_CLK_PER_SM} ex2 / clock / SM x "
+                                           f"{n_sms} SMs x {sm_mhz:.0f} MHz"},
+                    "hbm": hbm_part}
     else:
         roofline = {"bound": "hbm", "kernel": dom, "peak_source": peak_src, "traffic": traffic,
                     **hbm_part}
     step_bytes = wl.bytes_model(budget)
+    # this configuration's own floor: HBM bytes, the passes' contraction at
+    # the bf16 peak and their exponentials at the SFU peak (two passes over
+    # K unless a unit's logits fit in tensor memory)
+    passes = 1 if "window_stats" not in kernels else 2
+    floor = {"hbm_ms": step_bytes / (hbm * 1e9) * 1e3,
+             "tensor_ms": passes * flops / (tc_peak * 1e12) * 1e3,
+             "sfu_ms": passes * exps / sfu_peak * 1e3, "passes_over_K": passes}
+    bound = max(("hbm_ms", "tensor_ms", "sfu_ms"), key=lambda k: floor[k])
+    floor.update(bound=bound[:-3], ms=floor[bound], frac_of_floor=floor[bound] / ms)
 
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
@@ -433,35 +583,44 @@ def main():
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded, paper-shaped; no datasets)",
             "config": config_dict(wl, budget, world),
-            "gpu_launches": sum(n for _, n in prof.values()), "roofline": roofline, "kernels": kernels,
-            "clocks": clocks}
+            "gpu_launches": sum(n for _, n in prof.values()), "roofline": roofline,
+            "step_floor": floor, "kernels": kernels, "clocks": clocks}
+
+    # fresh input buffers every step: the TMA descriptors of the inputs are
+    # encoded and uploaded again on each call (a serving engine's KV buffers
+    # change from request to request)
+    if not args.no_extras:
+        x2 = workloads.Inputs(x.qwin.clone(), x.k.clone(), x.v.clone(), None)
+        sets = [x, x2]
+        step = [0]
+
+        def alternate():
+            xs = sets[step[0] & 1]
+            step[0] += 1
+            ctx.compress_all_layers(xs.qwin, xs.k, xs.v, budget, ko, vo, idx)
+
+        for _ in range(4):
+            alternate()
+        alt_ms = timed(alternate, args.steps, stream)
+        line["fresh_buffers_each_step"] = {
+            "ms_per_step": alt_ms, "extra_ms_per_step": alt_ms - ms,
+            "what": "two input sets in turn: every call encodes and uploads the TMA "
+                    "descriptors of its (request, layer) pairs"}
+        del x2, sets
 
     if not args.no_extras:
         # the same step when the prefill attention supplies the window rows'
         # softmax normalisers (no first pass over K)
-        lse = torch.empty((wl.requests, wl.layers, wl.q_heads, wl.window), dtype=torch.float32,
-                          device=dev)
-        pos = torch.arange(wl.seq_len, device=dev)
-        vis = pos[None, :] <= (wl.seq_len - wl.window + torch.arange(wl.window, device=dev))[:, None]
-        for r in range(wl.requests):
-            for l in range(wl.layers):
-                q = x.qwin[r, l].float().view(wl.kv_heads, wl.group, wl.window, wl.head_dim)
-                s_ = torch.einsum("hgwd,hnd->hgwn", q, x.k[r, l].float()) / wl.head_dim ** 0.5
-                lse[r, l] = torch.logsumexp(s_.masked_fill(~vis, float("-inf")), -1).reshape(
-                    wl.q_heads, wl.window)
-        del s_
+        lse, lse_src = fused_attention_lse(wl, x, dev)
+        torch.cuda.empty_cache()
         for _ in range(3):
             ctx.compress_with_lse(x.qwin, x.k, x.v, lse, budget, ko, vo, idx)
-        torch.cuda.synchronize()
-        g0 = torch.cuda.Event(enable_timing=True)
-        g1 = torch.cuda.Event(enable_timing=True)
-        g0.record(stream)
-        for _ in range(args.steps):
-            ctx.compress_with_lse(x.qwin, x.k, x.v, lse, budget, ko, vo, idx)
-        g1.record(stream)
-        torch.cuda.synchronize()
+        lse_ms = timed(lambda: ctx.compress_with_lse(x.qwin, x.k, x.v, lse, budget, ko, vo, idx),
+                       args.steps, stream)
         line["with_prefill_normalisers"] = {
-            "ms_per_step": g0.elapsed_time(g1) / args.steps,
+            "ms_per_step": lse_ms,
+            "step_roofline_frac": step_bytes / (lse_ms / 1e3) / 1e9 / hbm,
+            "normalisers_from": lse_src,
             "what": "bacon_compress_with_lse: the window rows' softmax normalisers come from the "
                     "prefill attention, so the first pass over K is skipped"}
         del lse
@@ -472,13 +631,8 @@ def main():
         sidx, slam = ctx.sweep(x.qwin, x.k, budget, variants)
         for _ in range(3):
             ctx.sweep(x.qwin, x.k, budget, variants, sidx, slam)
-        torch.cuda.synchronize()
-        g0.record(stream)
-        for _ in range(args.steps):
-            ctx.sweep(x.qwin, x.k, budget, variants, sidx, slam)
-        g1.record(stream)
-        torch.cuda.synchronize()
-        sweep_ms = g0.elapsed_time(g1) / args.steps
+        sweep_ms = timed(lambda: ctx.sweep(x.qwin, x.k, budget, variants, sidx, slam),
+                         args.steps, stream)
         line["ablation_sweep"] = {
             "variants": len(variants), "ms_per_sweep": sweep_ms,
             "ms_per_variant": sweep_ms / len(variants),
@@ -486,6 +640,16 @@ def main():
             "what": "bacon_sweep over the component ablation and the m / r sensitivity grid: "
                     "one set of window passes, then calibration and selection per variant"}
         del sidx, slam
+
+    # the timed step's selections at the oracle's sample units, and the inputs
+    # the oracle needs for them (host copies of layers 0-1)
+    want_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline
+    if want_cpu:
+        ctx.compress_all_layers(x.qwin, x.k, x.v, budget, ko, vo, idx)
+        ctx.sync()
+        gpu_idx = idx.cpu().numpy()
+        L2 = min(2, wl.layers)
+        host = tuple(workloads.bf16_bits(t[:, :L2]) for t in (x.qwin, x.k, x.v))
 
     # end to end through the host-buffer C call: H2D inputs, compress, D2H outputs
     if not args.no_e2e:
@@ -523,9 +687,10 @@ def main():
                                "uploaded, kept value rows read in place)"}
     ctx.close()
 
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(wl, budget)
+    if want_cpu:
+        line["cpu_baseline"] = cpu_baseline(wl, budget, host, gpu_idx)
     if rank == 0:
+        line["boundary_swaps"] = logged_swaps()
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()

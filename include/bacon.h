@@ -54,8 +54,10 @@
  * BACON_ETIMEOUT when a kernel's bounded pipeline wait (about a second) ran
  * out, after which the kernel drained its own work and returned, so the
  * context stays usable; BACON_EINVAL when bacon_compact was given an index
- * outside [0, seq_len).  A context must not be used from two threads at
- * once.
+ * outside [0, seq_len); BACON_ECUDA when an internal consistency check of a
+ * selection kernel failed (it emitted a different number of positions than
+ * its budget; never expected, its message says so).  A context must not be
+ * used from two threads at once.
  */
 #ifndef BACON_H
 #define BACON_H
@@ -319,15 +321,22 @@ bacon_status bacon_profile_read(bacon_ctx* ctx, double* ms, int* launches, int n
  * pointers, 16-byte aligned.  Limits: seq_len <= 16384,
  * q_heads * window <= 4096 and (q_heads / kv_heads) * window <= 512 (beyond
  * them: BACON_EUNSUPPORTED); malformed
- * arguments give BACON_EINVAL, a CUDA failure BACON_ECUDA.  No message is
- * recorded for bacon_last_error.
+ * arguments give BACON_EINVAL, a CUDA failure at launch BACON_ECUDA.  No
+ * message is recorded for bacon_last_error.  The status is returned before
+ * the kernels run, so an error found on the device (a bounded pipeline wait
+ * of about a second that ran out) is reported in the outputs instead: B_out,
+ * Q_out and E_out are then all NaN once the stream reaches the end of the
+ * call.  A caller that must tell this case apart checks one output value
+ * after synchronising.
  *
  * The first call on a device looks up the array's device address (with
  * that device current) and caches it; make that first call before any
  * stream capture.  Every call uses the same array: calls whose work can
  * overlap on the GPU (different streams, or several host threads) race and
- * must be serialised by the caller.  Nothing in the array has to start at
- * zero: each call writes every entry it later reads. */
+ * must be serialised by the caller.  The array keeps the last call's
+ * contents; its error word, the one entry that must start at zero, is
+ * cleared by each call on its stream, and every other entry a call reads
+ * it has written first. */
 bacon_status bacon_window_scores_noalloc(int kv_heads, int q_heads, int head_dim, int window,
                                          const void* q_win, const void* k, int seq_len,
                                          float* B_out, float* Q_out, float* E_out,

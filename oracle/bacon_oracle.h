@@ -12,7 +12,8 @@
  *   - the observation window W is the last W prompt positions N-W .. N-1,
  *     the last query position D is N-1;
  *   - a kv-head h serves G = Hq/Hkv query heads; their window attention rows
- *     are averaged into the head's score (GQA reading, see DESIGN notes);
+ *     are averaged into the head's score (the paper does not address GQA;
+ *     this is the reading both the oracle and the CUDA path follow);
  *   - every floating-point quantity is double; bf16 inputs are widened
  *     exactly.
  */

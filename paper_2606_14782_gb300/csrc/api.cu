@@ -1172,10 +1172,15 @@ bacon_status bacon_sync(bacon_ctx* ctx, bacon_stream stream)
     int flag = 0;
     BACON_CUDA(cudaMemcpy(&flag, ctx->err, sizeof(int), cudaMemcpyDeviceToHost), "error flag read");
     if (flag) {
-        cudaMemset(ctx->err, 0, sizeof(int));
+        // the word is cleared before the latched error is reported, so that
+        // the context's next call starts clean
+        BACON_CUDA(cudaMemset(ctx->err, 0, sizeof(int)), "error flag reset");
         if (flag == 1) return fail(BACON_EINVAL, "a gather index was outside [0, seq_len)");
         if (flag == 3) return fail(BACON_ETIMEOUT, "a window-score kernel timed out waiting on its pipeline");
-        return fail(BACON_ECUDA, "device selection check failed (code %d)", flag);
+        if (flag == 2)
+            return fail(BACON_ECUDA, "internal check failed: a selection emitted a different count "
+                                     "than its budget");
+        return fail(BACON_ECUDA, "unknown device error code %d", flag);
     }
     return BACON_OK;
 }

@@ -8,6 +8,15 @@
 // their scratch (pass-1 partial statistics, the per-row normalisers and the
 // two TMA descriptors) in one file-scope __device__ array instead of
 // context-owned buffers.
+//
+// The call returns before its kernels run, so a device-side failure (a
+// bounded pipeline wait that ran out) cannot come back as its status.  The
+// same array holds an error word for that: each call clears it, the window
+// kernels latch a timeout in it, and a last small kernel fills B, Q and E
+// with NaN when it is set, so that a caller never reads partial scores as
+// valid ones.
+#include <atomic>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 
@@ -26,16 +35,47 @@ constexpr int kMaxChunks = kMaxSeq / kChunk;
 constexpr int kMaxDevices = 64;
 
 constexpr int kMapBytes = 2 * sizeof(CUtensorMap);  // K map, window-query map
+constexpr int kErrSlots = 2;                        // 16 bytes holding the error word
 
 // [units][chunks][rows] partial (max, sum) pairs, then [units][rows] fp32
-// normalisers packed two per float2, then the two 128-byte TMA descriptors.
-// 528.25 KiB, held by every GPU that loads the library until the process
-// exits.
+// normalisers packed two per float2, then the two 128-byte TMA descriptors,
+// then the device error word.  About 528 KiB, held by every GPU that loads
+// the library until the process exits.
 static __device__ __align__(256) float2
-    g_scratch[kMaxTotalRows * kMaxChunks + kMaxTotalRows / 2 + kMapBytes / sizeof(float2)];
+    g_scratch[kMaxTotalRows * kMaxChunks + kMaxTotalRows / 2 + kMapBytes / sizeof(float2) +
+              kErrSlots];
 
 std::mutex g_setup_mutex;
 void* g_scratch_addr[kMaxDevices] = {};
+
+// Test-only fault injection: when BACON_FAULT=missing_arrival is set at the
+// first call of the process, that call's pass 1 withholds one K-tile load,
+// so its bounded waits run out (nothing faults).  -1 = not read yet.
+std::atomic<int> g_fault_pending{-1};
+
+int take_fault()
+{
+    int s = g_fault_pending.load();
+    if (s < 0) {
+        const char* f = std::getenv("BACON_FAULT");
+        g_fault_pending.compare_exchange_strong(s, (f && std::strcmp(f, "missing_arrival") == 0) ? 1 : 0);
+    }
+    int one = 1;
+    return g_fault_pending.compare_exchange_strong(one, 0) ? 1 : 0;
+}
+
+// B, Q and E become NaN when a window kernel of this call latched an error.
+__global__ void poison_on_error_kernel(const int* err, float* B, float* Q, float* E, size_t n)
+{
+    if (*reinterpret_cast<const volatile int*>(err) == 0) return;
+    const float nan = __int_as_float(0x7fc00000);
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (size_t)gridDim.x * blockDim.x) {
+        B[i] = nan;
+        Q[i] = nan;
+        E[i] = nan;
+    }
+}
 
 }  // namespace
 
@@ -88,6 +128,8 @@ bacon_status bacon_window_scores_noalloc(int kv_heads, int q_heads, int head_dim
     float* lse2 = reinterpret_cast<float*>(scratch + (size_t)kMaxTotalRows * kMaxChunks);
     CUtensorMap* maps =
         reinterpret_cast<CUtensorMap*>(scratch + (size_t)kMaxTotalRows * kMaxChunks + kMaxTotalRows / 2);
+    int* err = reinterpret_cast<int*>(scratch + (size_t)kMaxTotalRows * kMaxChunks +
+                                      kMaxTotalRows / 2 + kMapBytes / sizeof(float2));
     // descriptors are encoded on the host and copied from this stack buffer;
     // a copy from pageable memory is staged before cudaMemcpyAsync returns
     alignas(64) CUtensorMap host_maps[2];
@@ -97,6 +139,8 @@ bacon_status bacon_window_scores_noalloc(int kv_heads, int q_heads, int head_dim
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (cudaMemcpyAsync(maps, host_maps, sizeof host_maps, cudaMemcpyHostToDevice, st) != cudaSuccess)
         return BACON_ECUDA;
+    // the error word must start at zero for this call
+    if (cudaMemsetAsync(err, 0, sizeof(int), st) != cudaSuccess) return BACON_ECUDA;
     TcArgs a;
     a.kmaps = maps;
     a.qmaps = maps + 1;
@@ -108,10 +152,19 @@ bacon_status bacon_window_scores_noalloc(int kv_heads, int q_heads, int head_dim
     a.B = B_out;
     a.Q = Q_out;
     a.E = E_out;
-    a.err = nullptr;
-    cudaError_t e = launch_window_stats_tc(a, st);
+    a.err = err;
+    TcArgs a1 = a;
+    a1.fault = take_fault();
+    cudaError_t e = launch_window_stats_tc(a1, st);
     if (e == cudaSuccess) e = launch_window_combine(s, chunks, partial, lse2, st);
     if (e == cudaSuccess) e = launch_window_scores_tc(a, st);
+    if (e == cudaSuccess) {
+        const size_t n = (size_t)kv_heads * seq_len;
+        const size_t blocks = (n + 255) / 256;
+        poison_on_error_kernel<<<(unsigned)(blocks < 1024 ? blocks : 1024), 256, 0, st>>>(
+            err, B_out, Q_out, E_out, n);
+        e = cudaGetLastError();
+    }
     return e == cudaSuccess ? BACON_OK : BACON_ECUDA;
 }
 

@@ -60,8 +60,11 @@ __device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist
     }
     __syncthreads();
     if (warp == 0) {
-        const uint32_t a = __reduce_min_sync(0xffffffffu, (uint32_t)hist[lane]);
-        const uint32_t b = __reduce_max_sync(0xffffffffu, (uint32_t)hist[32 + lane]);
+        // only the first nwarps entries were written: the other lanes take
+        // the neutral element of each reduction
+        const bool held = lane < (int)(blockDim.x >> 5);
+        const uint32_t a = __reduce_min_sync(0xffffffffu, held ? (uint32_t)hist[lane] : 0xffffffffu);
+        const uint32_t b = __reduce_max_sync(0xffffffffu, held ? (uint32_t)hist[32 + lane] : 0u);
         if (lane == 0) {
             bcast[0] = (int)a;
             bcast[1] = (int)b;

@@ -25,3 +25,17 @@ def pytest_collection_modifyitems(config, items):
     for item in items:
         if "gpu" in item.keywords:
             item.add_marker(skip)
+
+
+def pytest_sessionfinish(session, exitstatus):
+    """Writes the session's boundary-swap log (tests/parity.py) to the path in
+    BACON_SWAP_LOG, keyed by a digest of the kernels' sources."""
+    if not os.environ.get("BACON_SWAP_LOG"):
+        return
+    import parity
+    if not parity.SWAP_LOG:
+        return
+    import bench
+    csrc = os.path.join(ROOT, "paper_2606_14782_gb300", "csrc")
+    names = sorted(n for n in os.listdir(csrc) if n.endswith((".cu", ".cuh", ".h")))
+    parity.write_swap_log(bench.source_digest(names))

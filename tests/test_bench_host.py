@@ -91,9 +91,51 @@ def test_reference_arm_json_line():
 
 
 def test_cpu_baseline_reports_threads_and_one_thread():
+    import numpy as np
+
+    import oracle
     from paper_2606_14782_gb300 import workloads
     wl = workloads.CONFIGS["tiny"]
-    cb = bench.cpu_baseline(wl, wl.budgets[0])
+    x = workloads.generate(wl, seed=0, device="cpu")
+    host = tuple(workloads.bf16_bits(t) for t in (x.qwin, x.k, x.v))
+    # the oracle's own selections stand in for the GPU's: no swaps
+    ref = oracle.compress(*host, wl.budgets[0], oracle.Params(pool_kernel=wl.pool))
+    idx = np.stack([np.stack([ref[(0, l, h)]["idx"] for h in range(wl.kv_heads)])
+                    for l in range(wl.layers)])[None]
+    cb = bench.cpu_baseline(wl, wl.budgets[0], host, idx)
     assert cb["kind"] == "oracle" and cb["unit"] == bench.UNIT and cb["value"] > 0
     assert cb["cores"] == min(os.cpu_count() or 1, wl.requests * wl.kv_heads)
     assert cb["single_thread"]["cores"] == 1 and cb["single_thread"]["value"] > 0
+    chk = cb["sample_selection_check"]
+    assert chk["boundary_swaps"] == 0 and chk["all_within_band"] and chk["units"] == 2 * 4
+
+
+def test_boundary_swap_count_and_band():
+    import numpy as np
+    N, W, budget = 12, 2, 6          # 10 candidates, 4 selected
+    S = np.array([9, 8, 7, 5, 5.00001, 1, 0, 0, 0, 0, 0, 0], dtype=np.float64)
+    orc = np.array([0, 1, 2, 4, 10, 11])
+    # position 3 instead of 4: within the band around the boundary score 5
+    assert bench.boundary_swaps(np.array([0, 1, 2, 3, 10, 11]), orc, S, N, W, budget) == (1, True)
+    # position 5 instead of 4: far below the boundary
+    assert bench.boundary_swaps(np.array([0, 1, 2, 5, 10, 11]), orc, S, N, W, budget) == (1, False)
+    assert bench.boundary_swaps(orc, orc, S, N, W, budget) == (0, True)
+
+
+def test_logged_swaps_reads_the_parity_log(tmp_path):
+    csrc = os.path.join(ROOT, "paper_2606_14782_gb300", "csrc")
+    names = sorted(n for n in os.listdir(csrc) if n.endswith((".cu", ".cuh", ".h")))
+    doc = {"code_sha256_16": bench.source_digest(names),
+           "cases": {"gui B=1024": {"swaps": 3, "units_checked": 448, "selected_per_unit": 960,
+                                    "max_gap_over_band": 0.5},
+                     "edge ragged B=100": {"swaps": 0, "units_checked": 8,
+                                           "selected_per_unit": 68, "max_gap_over_band": 0}}}
+    path = tmp_path / "swaps.json"
+    path.write_text(json.dumps(doc))
+    got = bench.logged_swaps(str(path))
+    assert got["current_code"] is True
+    assert got["cases"] == {"gui B=1024": {"swaps": 3, "units": 448, "selected_per_unit": 960,
+                                           "max_gap_over_band": 0.5}}
+    doc["code_sha256_16"] = "0" * 16
+    path.write_text(json.dumps(doc))
+    assert bench.logged_swaps(str(path))["current_code"] is False

@@ -20,8 +20,7 @@ import pytest
 import torch
 
 from paper_2606_14782_gb300 import bacon, build, workloads
-from parity import check_scores
-from test_gpu_parity import compare, oracle_run, prefill_lse, run_gpu
+from test_gpu_parity import compare, oracle_run, prefill_lse, run_gpu, run_with_lse
 
 pytestmark = pytest.mark.gpu
 
@@ -73,7 +72,7 @@ def test_random_shapes(name, over, budget):
     x = workloads.generate(wl, seed=11, device="cuda")
     gpu = run_gpu(wl, x, budget)
     orc = oracle_run(wl, x, budget)
-    compare(wl, x, budget, gpu, orc)
+    compare(wl, x, budget, gpu, orc, case=f"fuzz {name} B={budget}")
     # each window softmax row sums to one, so B and Q do per unit
     np.testing.assert_allclose(gpu["B"].sum(-1), 1.0, atol=2e-4)
     np.testing.assert_allclose(gpu["Q"].sum(-1), 1.0, atol=2e-4)
@@ -103,15 +102,10 @@ def test_random_shapes_layer_path(name, over, budget):
 
 @pytest.mark.parametrize("name,over,budget", SHAPES, ids=[s[0] for s in SHAPES])
 def test_random_shapes_prefill_normalisers(name, over, budget):
+    """The one-pass path given the prefill's normalisers, against the oracle."""
     wl = workloads.CONFIGS["tiny"].with_(**over)
     x = workloads.generate(wl, seed=11, device="cuda")
-    whole = run_gpu(wl, x, budget)
-    p = bacon.default_params(keep_scores=1, max_seq_len=wl.seq_len, max_requests=wl.requests)
-    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool,
-                        budget, params=p)
-    ctx.compress_with_lse(x.qwin, x.k, x.v, prefill_lse(wl, x), budget)
-    ctx.sync()
-    shp = (wl.requests, wl.layers, wl.kv_heads, wl.seq_len)
-    for kind in ("B", "Q", "E"):
-        check_scores(f"{name} {kind}", ctx.scores(kind).cpu().numpy().reshape(shp), whole[kind])
-    ctx.close()
+    gpu = run_with_lse(wl, x, prefill_lse(wl, x), budget)
+    orc = oracle_run(wl, x, budget)
+    compare(wl, x, budget, gpu, orc, case=f"fuzz {name} B={budget} normalisers from the prefill",
+            path="bacon_compress_with_lse")
