@@ -6,11 +6,23 @@
 //   S = B~ + lambda V                                 (Eq. 16)
 //   the K best candidates by S, ascending, then the window (Eq. 17)
 // Both "best k" sets use one order: larger value first, equal values ->
-// lower position first (select.cuh: range-adaptive radix select, then
-// index-ordered warp-segmented sweeps that resolve ties and emit ascending
-// positions).  The two standard deviations come from one sweep that sums
-// moments about fixed shifts in fp32 (the shifts keep the differences
-// small, so no precision is lost to cancellation).
+// lower position first.  A range-adaptive radix select (select.cuh) finds
+// the k-th best key and how many of the keys equal to it are taken; the
+// members are then decided thread by thread in position order.
+//
+// Each thread owns PER consecutive positions [t PER, t PER + PER), so the
+// pooling and coherence windows slide along a thread's own positions and
+// the position order of the members is (thread, slot) order: one
+// block-wide exclusive scan gives every thread its tie rank or its output
+// offset.  The per-position arrays in shared memory are stored slot-major,
+// element (slot k, thread t) at k T + t: when every thread of a warp reads
+// its own position plus the same offset, the 32 reads fall in consecutive
+// words (no bank conflicts), and the radix select's passes, which walk the
+// storage index s = k T + t, read consecutive words as well.
+//
+// The two standard deviations come from one walk that sums moments about
+// fixed shifts in fp32 (the shifts keep the differences small, so no
+// precision is lost to cancellation).
 #include "common.cuh"
 #include "select.cuh"
 
@@ -19,14 +31,14 @@ namespace {
 
 using namespace sel;
 
-// Threads per CTA and tokens per thread depend on the prompt length only
+// Threads per CTA and positions per thread depend on the prompt length only
 // (so that every call on the same shape reduces in the same order and gives
-// the same bits): 256 threads of up to 8 tokens up to 2048 tokens, where
-// several CTAs share an SM; 1024 threads of up to 16 tokens up to 16384
-// tokens; 1024 threads of up to kMaxPer tokens above.
-constexpr int kMaxPer = 24;
+// the same bits): 256 threads of 8 positions up to 2048 tokens, where
+// several CTAs share an SM; 1024 threads of 16 positions up to 16384
+// tokens; 1024 threads of 24 above (up to 24576).
 constexpr int kSmallPrompt = 2048;
-constexpr int kMidPrompt = 16384;  // 1024 threads x 16 tokens
+constexpr int kMidPrompt = 16384;
+constexpr int kMaxPrompt = 24576;
 
 // Block-wide fp32 sum by a shuffle tree (pairwise, so the rounding error
 // grows with log2 of the count).  FP64 is avoided: its rate on this part is
@@ -81,6 +93,37 @@ __device__ float4 block_sum4(float4 v, float* red)
     return tot;
 }
 
+// Exclusive prefix sum of one int per thread, in thread order; *total
+// receives the sum.  warp_sums holds 32 ints.
+__device__ int block_exclusive_scan(int v, int* warp_sums, int* total)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) warp_sums[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        const int nw = (int)(blockDim.x >> 5);
+        const int w = lane < nw ? warp_sums[lane] : 0;
+        int wi = w;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, wi, o);
+            if (lane >= o) wi += y;
+        }
+        if (lane < nw) warp_sums[lane] = wi - w;
+        if (lane == 31) *total = wi;
+    }
+    __syncthreads();
+    const int r = warp_sums[warp] + incl - v;
+    __syncthreads();
+    return r;
+}
+
 // Ask L2 to fetch the n floats at p (one prefetch per 128-byte line, every
 // address inside the array), so that later loads of them hit L2.
 __device__ __forceinline__ void prefetch_l2(const float* p, int n)
@@ -89,42 +132,120 @@ __device__ __forceinline__ void prefetch_l2(const float* p, int n)
         asm volatile("prefetch.global.L2 [%0];" ::"l"(p + i));
 }
 
-// dst[0, n) = src[0, n) with independent 16-byte loads (n % 4 == 0 and both
-// 16-byte aligned), so the copy costs a few memory round trips, not one per
-// element.
-__device__ __forceinline__ void stage(float* dst, const float* src, int n)
+// x[k] = src[i0 + k] for the thread's PER positions (0 at and past n), with
+// 16-byte loads when the run is whole and aligned (n % 4 == 0).
+template <int PER>
+__device__ __forceinline__ void load_run(const float* __restrict__ src, int i0, int n, float* x)
 {
-    const float4* s4 = reinterpret_cast<const float4*>(src);
-    float4* d4 = reinterpret_cast<float4*>(dst);
-    const int n4 = n >> 2;
-    for (int i = threadIdx.x; i < n4; i += 4 * blockDim.x) {
-        float4 v[4];
+    if ((n & 3) == 0 && i0 + PER <= n) {
+        const float4* s4 = reinterpret_cast<const float4*>(src + i0);
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-            if (i + k * (int)blockDim.x < n4) v[k] = __ldg(s4 + i + k * blockDim.x);
+        for (int q = 0; q < PER / 4; ++q) {
+            const float4 v = __ldg(s4 + q);
+            x[4 * q] = v.x;
+            x[4 * q + 1] = v.y;
+            x[4 * q + 2] = v.z;
+            x[4 * q + 3] = v.w;
+        }
+    } else {
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-            if (i + k * (int)blockDim.x < n4) d4[i + k * blockDim.x] = v[k];
+        for (int k = 0; k < PER; ++k) x[k] = i0 + k < n ? src[i0 + k] : 0.f;
     }
+}
+
+// dst[i0 + k] = x[k] for the positions below n.
+template <int PER>
+__device__ __forceinline__ void store_run(float* dst, int i0, int n, const float* x)
+{
+    if ((n & 3) == 0 && i0 + PER <= n) {
+        float4* d4 = reinterpret_cast<float4*>(dst + i0);
+#pragma unroll
+        for (int q = 0; q < PER / 4; ++q)
+            d4[q] = make_float4(x[4 * q], x[4 * q + 1], x[4 * q + 2], x[4 * q + 3]);
+    } else {
+#pragma unroll
+        for (int k = 0; k < PER; ++k)
+            if (i0 + k < n) dst[i0 + k] = x[k];
+    }
+}
+
+// Slot-major shared-memory array of T threads x PER positions.
+template <int T, int PER>
+struct Slots {
+    float* a;
+    // storage index of position i, and the position held at storage index s
+    __device__ static __forceinline__ int at(int i) { return (i % PER) * T + i / PER; }
+    __device__ static __forceinline__ int pos(int s) { return (s % T) * PER + s / T; }
+    __device__ __forceinline__ float& own(int k) const { return a[k * T + (int)threadIdx.x]; }
+    __device__ __forceinline__ float operator[](int i) const { return a[at(i)]; }
+};
+
+// Keys of the candidates [0, n_cand) of a slot-major array, walked by
+// storage index (the radix select's passes read consecutive words).
+template <int T, int PER>
+struct SlotKeys {
+    const float* a;
+    int n_cand;
+    __device__ __forceinline__ bool operator()(int s, uint32_t& key) const
+    {
+        if (Slots<T, PER>::pos(s) >= n_cand) return false;
+        key = float_key(a[s]);
+        return true;
+    }
+};
+
+// Membership of the thread's candidates in the k best (bit k of the result):
+// key > tau, or key == tau among the first `need` such keys in position
+// order.  eq_before = keys equal to tau at lower positions (other threads).
+template <int T, int PER>
+__device__ __forceinline__ uint32_t members(const Slots<T, PER>& arr, int i0, int n_cand,
+                                            const SelectResult& sel, int eq_before)
+{
+    uint32_t m = 0u;
+    int rank = eq_before;
+#pragma unroll
+    for (int k = 0; k < PER; ++k) {
+        if (i0 + k < n_cand) {
+            const uint32_t key = float_key(arr.own(k));
+            const bool eq = key == sel.tau;
+            if (key > sel.tau || (eq && rank < sel.need)) m |= 1u << k;
+            rank += eq;
+        }
+    }
+    return m;
+}
+
+// Keys equal to tau at lower positions than this thread's run (0 without a
+// scan when every tie is taken: membership then never needs the rank).
+template <int T, int PER>
+__device__ __forceinline__ int ties_before(const Slots<T, PER>& arr, int i0, int n_cand,
+                                           const SelectResult& sel, int* warp_sums, int* total)
+{
+    if (sel.all_ties_in()) return 0;
+    int eq = 0;
+#pragma unroll
+    for (int k = 0; k < PER; ++k)
+        eq += (i0 + k < n_cand) && float_key(arr.own(k)) == sel.tau;
+    return block_exclusive_scan(eq, warp_sums, total);
 }
 
 // One unit (request, layer, kv-head) u under hyper-parameters c.  lam_out
 // (may be null) receives lambda; idx_pair is the pair's [Hkv][kept] output.
-// PER bounds the tokens per thread (N <= PER blockDim.x).
-template <int PER>
+// N <= T PER.
+template <int T, int PER>
 __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, const CalibArgs& a,
                                                int u, float* lam_out, int32_t* idx_pair)
 {
     extern __shared__ __align__(16) float sm[];
-    const int N = s.N, W = s.W;
-    float* Sb = sm;      // pooled backbone B~, then the final score S
-    float* Vs = sm + N;  // calibrated evidence V
+    const Slots<T, PER> A1{sm};            // B (pooling), then E (coherence)
+    const Slots<T, PER> A2{sm + T * PER};  // pooled backbone B~, then the final score S
     __shared__ int hist[kSelHist];
     __shared__ int bcast[8];
     __shared__ int warp_sums[32];
     __shared__ float red[4 * 33];
     __shared__ int total_s;
 
+    const int N = s.N, W = s.W;
     const int pair = u / s.hkv, h = u - pair * s.hkv;
     const int rq = pair / s.layers;
     const int layer = a.layer0 + (pair - rq * s.layers);
@@ -132,6 +253,7 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
     const int n_cand = N - win;
     const int kept_total = min(a.budget[pair], N);
     const int keep = kept_total - win;
+    const int i0 = (int)threadIdx.x * PER;
 
     uint32_t skmin = 0xffffffffu, skmax = 0u;  // key range of S over the candidates
     auto Eof = [&](int j) -> const float* {
@@ -142,112 +264,145 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
     if (a.compute_scores) {
         const float* Bu = a.B + (size_t)u * N;
         const float* Ec = Eof(layer);
-        const int half = c.pool / 2;
         const int nprev = min(c.m, layer);
         const float inv_prev = nprev > 0 ? 1.f / (float)nprev : 0.f;
-        // the residuals of this layer and of the preceding ones are read
-        // only after the pooling: start bringing them into L2 now
+        // the residuals are read only after the pooling: start bringing them
+        // into L2 now
         prefetch_l2(Ec, N);
         if (c.use_T)
             for (int j = layer - nprev; j < layer; ++j) prefetch_l2(Eof(j), N);
-        // B -> Vs (staging), then the pooled backbone over the candidates -> Sb
-        if ((N & 3) == 0)
-            stage(Vs, Bu, N);
-        else
-            for (int i = threadIdx.x; i < N; i += blockDim.x) Vs[i] = Bu[i];
+
+        // ---- pooled backbone over the candidates (max over [i - half, i + half])
+        float x[PER];
+        load_run<PER>(Bu, i0, N, x);
+#pragma unroll
+        for (int k = 0; k < PER; ++k) A1.own(k) = x[k];
         __syncthreads();
         uint32_t kmin = 0xffffffffu, kmax = 0u;  // key range of B~ over the candidates
-        for (int i = threadIdx.x; i < N; i += blockDim.x) {
-            float mx = 0.f;
-            if (i < n_cand) {
-                mx = -INFINITY;
-                const int lo = max(0, i - half), hi = min(n_cand - 1, i + half);
-#pragma unroll 4
-                for (int v = lo; v <= hi; ++v) mx = fmaxf(mx, Vs[v]);
-                kmin = min(kmin, float_key(mx));
-                kmax = max(kmax, float_key(mx));
-            }
-            Sb[i] = mx;
-        }
-        __syncthreads();
-        // E -> Vs (staging); V is built in registers, then written over it
-        if ((N & 3) == 0)
-            stage(Vs, Ec, N);
-        else
-            for (int i = threadIdx.x; i < N; i += blockDim.x) Vs[i] = Ec[i];
-        __syncthreads();
-        float vreg[PER];
-        // persistence: mean of E over the preceding min(m, l) layers (Eqs. 8-9)
+        const int half = c.pool / 2;
+        if (half == 3) {
+            // width 7 (the default): the run and three positions either side
+            // in registers, each output a maximum of seven by three max3
+            float w[PER + 6];
 #pragma unroll
-        for (int k = 0; k < PER; ++k) vreg[k] = 0.f;
+            for (int m = 0; m < 3; ++m) {
+                const int jl = i0 - 3 + m, jr = i0 + PER + m;
+                w[m] = (jl >= 0 && jl < n_cand) ? A1[jl] : -INFINITY;
+                w[PER + 3 + m] = jr < n_cand ? A1[jr] : -INFINITY;
+            }
+#pragma unroll
+            for (int k = 0; k < PER; ++k) w[3 + k] = i0 + k < n_cand ? x[k] : -INFINITY;
+#pragma unroll
+            for (int k = 0; k < PER; ++k) {
+                float mx = 0.f;
+                if (i0 + k < n_cand) {
+                    mx = max3f(max3f(w[k], w[k + 1], w[k + 2]),
+                                 max3f(w[k + 3], w[k + 4], w[k + 5]), w[k + 6]);
+                    kmin = min(kmin, float_key(mx));
+                    kmax = max(kmax, float_key(mx));
+                }
+                A2.own(k) = mx;
+            }
+        } else {
+#pragma unroll
+            for (int k = 0; k < PER; ++k) {
+                const int i = i0 + k;
+                float mx = 0.f;
+                if (i < n_cand) {
+                    mx = -INFINITY;
+                    const int lo = max(0, i - half), hi = min(n_cand - 1, i + half);
+                    for (int v = lo; v <= hi; ++v) mx = fmaxf(mx, A1[v]);
+                    kmin = min(kmin, float_key(mx));
+                    kmax = max(kmax, float_key(mx));
+                }
+                A2.own(k) = mx;
+            }
+        }
+
+        // ---- persistence: mean of E over the preceding min(m, l) layers (Eqs. 8-9)
+        float v[PER];
+#pragma unroll
+        for (int k = 0; k < PER; ++k) v[k] = 0.f;
         if (c.use_T) {
             for (int j = layer - nprev; j < layer; ++j) {
-                const float* Ej = Eof(j);
-                // every load in flight at once: indices past the end are
-                // clamped to the last token (in bounds) and their values
-                // dropped
-                float x[PER];
+                float e[PER];
+                load_run<PER>(Eof(j), i0, N, e);
 #pragma unroll
-                for (int k = 0; k < PER; ++k) x[k] = Ej[min((int)threadIdx.x + k * (int)blockDim.x, N - 1)];
-#pragma unroll
-                for (int k = 0; k < PER; ++k)
-                    if ((int)threadIdx.x + k * (int)blockDim.x < N) vreg[k] += x[k];
+                for (int k = 0; k < PER; ++k) v[k] += e[k];
             }
+#pragma unroll
+            for (int k = 0; k < PER; ++k) v[k] *= inv_prev;
         }
+        __syncthreads();  // every pooling read of A1 is done
+        load_run<PER>(Ec, i0, N, x);
 #pragma unroll
         for (int k = 0; k < PER; ++k) {
-            const int i = threadIdx.x + k * blockDim.x;
-            if (i < N) {
-                // coherence: truncated radius-r box mean of E (Eqs. 5-7)
-                const int lo = max(0, i - c.r), hi = min(N - 1, i + c.r);
-                float sum = 0.f;
-#pragma unroll 4
-                for (int v = lo; v <= hi; ++v) sum += Vs[v];
-                const float L = sum / (float)(hi - lo + 1);
-                float V = 0.f;
-                if (c.use_E) V += Vs[i];
-                if (c.use_L) V += L;
-                if (c.use_T) V += vreg[k] * inv_prev;
-                vreg[k] = V;
-            }
+            A1.own(k) = x[k];
+            if (c.use_E) v[k] += x[k];
         }
         __syncthreads();
+        // ---- coherence: truncated radius-r box mean of E (Eqs. 5-7), the
+        // window sum sliding along the run
+        if (c.use_L) {
+            const int r = c.r;
+            int lo = max(0, i0 - r), hi = min(N - 1, i0 + r);
+            float sum = 0.f;
+            for (int j = lo; j <= hi; ++j) sum += A1[j];
+#pragma unroll
+            for (int k = 0; k < PER; ++k) {
+                const int i = i0 + k;
+                if (i < N) {
+                    // the window sum of non-negative values: rounding in the
+                    // slide can leave ~1e-9 below zero after a large value
+                    // leaves the window, so it is clamped
+                    v[k] += fmaxf(sum, 0.f) / (float)(hi - lo + 1);
+                    // the window of i + 1: drop i - r, add i + 1 + r
+                    if (i - r >= 0) sum -= A1[i - r];
+                    if (i + 1 + r <= N - 1) sum += A1[i + 1 + r];
+                    lo = max(0, i + 1 - r);
+                    hi = min(N - 1, i + 1 + r);
+                }
+            }
+        }
         float vsum = 0.f;  // over the candidates: the shift of the moments below
 #pragma unroll
         for (int k = 0; k < PER; ++k) {
-            const int i = threadIdx.x + k * blockDim.x;
-            if (i < N) Vs[i] = vreg[k];
-            if (i < n_cand) vsum += vreg[k];
+            if (i0 + k >= N) v[k] = 0.f;
+            if (i0 + k < n_cand) vsum += v[k];
         }
-        __syncthreads();
-        if (a.V) for (int i = threadIdx.x; i < N; i += blockDim.x) a.V[(size_t)u * N + i] = Vs[i];
-        if (a.Bp) for (int i = threadIdx.x; i < N; i += blockDim.x) a.Bp[(size_t)u * N + i] = Sb[i];
+        if (a.V) store_run<PER>(a.V + (size_t)u * N, i0, N, v);
+        if (a.Bp) {
+#pragma unroll
+            for (int k = 0; k < PER; ++k) x[k] = A2.own(k);
+            store_run<PER>(a.Bp + (size_t)u * N, i0, N, x);
+        }
 
-        // Eqs. 12-15
+        // ---- Eqs. 12-15
         const int calib_keep = min(a.calib_budget[pair], N) - win;
         const long long Ml = (long long)c.rho * (long long)(calib_keep > 0 ? calib_keep : 0);
         const int M = (int)(Ml < n_cand ? Ml : n_cand);
         float lam = 0.f;
         if (M > 0) {
-            const SelectResult sel =
-                radix_select_range(n_cand, M, FloatKeys{Sb}, hist, bcast, kmin, kmax);
-            const Segment sg = warp_segment(n_cand);
-            const int eqb = eq_before_segment(Sb, sg, sel, warp_sums, &total_s);
+            const SelectResult sel = radix_select_range(T * PER, M, SlotKeys<T, PER>{A2.a, n_cand},
+                                                        hist, bcast, kmin, kmax);
+            const int eqb = ties_before(A2, i0, n_cand, sel, warp_sums, &total_s);
+            const uint32_t mem = members(A2, i0, n_cand, sel, eqb);
             // moments about fixed shifts in one walk: B~ about its M-th value,
             // V about its mean over the candidates (both near the members'
             // means, so the fp32 differences keep their precision)
             const float pb = key_float(sel.tau);
             const float pv = block_sum(vsum, red) / (float)n_cand;
             float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-            walk_topk(Sb, sg, sel, eqb, [&](int i, bool, bool in) {
-                if (in) {
-                    const float db = Sb[i] - pb, dv = Vs[i] - pv;
+#pragma unroll
+            for (int k = 0; k < PER; ++k) {
+                if ((mem >> k) & 1u) {
+                    const float db = A2.own(k) - pb, dv = v[k] - pv;
                     acc.x += db;
                     acc.y = fmaf(db, db, acc.y);
                     acc.z += dv;
                     acc.w = fmaf(dv, dv, acc.w);
                 }
-            });
+            }
             const float4 tot = block_sum4(acc, red);
             const float inv_m = 1.f / (float)M;
             const float mb = tot.x * inv_m, mv = tot.z * inv_m;
@@ -256,63 +411,48 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
             lam = c.gamma * stdb / (stdv + c.eps);
         }
         if (threadIdx.x == 0 && lam_out) *lam_out = lam;
-        kmin = 0xffffffffu;
-        kmax = 0u;
-        for (int i = threadIdx.x; i < n_cand; i += blockDim.x) {
-            const float sv = fmaf(lam, Vs[i], Sb[i]);
-            Sb[i] = sv;
-            kmin = min(kmin, float_key(sv));
-            kmax = max(kmax, float_key(sv));
+        // ---- Eq. 16 over the candidates (0 elsewhere)
+#pragma unroll
+        for (int k = 0; k < PER; ++k) {
+            float sv = 0.f;
+            if (i0 + k < n_cand) {
+                sv = fmaf(lam, v[k], A2.own(k));
+                skmin = min(skmin, float_key(sv));
+                skmax = max(skmax, float_key(sv));
+            }
+            A2.own(k) = sv;
+            x[k] = sv;
         }
-        skmin = kmin;
-        skmax = kmax;
+        if (a.write_S) store_run<PER>(a.S + (size_t)u * N, i0, N, x);
         __syncthreads();
-        if (a.write_S)
-            for (int i = threadIdx.x; i < N; i += blockDim.x) a.S[(size_t)u * N + i] = Sb[i];
     } else {
-        for (int i = threadIdx.x; i < N; i += blockDim.x) Sb[i] = a.S[(size_t)u * N + i];
+        float x[PER];
+        load_run<PER>(a.S + (size_t)u * N, i0, N, x);
+#pragma unroll
+        for (int k = 0; k < PER; ++k) {
+            A2.own(k) = x[k];
+            if (i0 + k < n_cand) {
+                skmin = min(skmin, float_key(x[k]));
+                skmax = max(skmax, float_key(x[k]));
+            }
+        }
         __syncthreads();
     }
 
     if (!a.do_select) return;
-    if (!a.compute_scores)
-        for (int i = threadIdx.x; i < n_cand; i += blockDim.x) {
-            skmin = min(skmin, float_key(Sb[i]));
-            skmax = max(skmax, float_key(Sb[i]));
-        }
+    // ---- Eq. 17: the K best candidates by S, ascending, then the window
     int32_t* out = idx_pair + (size_t)h * kept_total;
     if (keep >= n_cand) {
         for (int i = threadIdx.x; i < n_cand; i += blockDim.x) out[i] = i;
     } else if (keep > 0) {
-        const SelectResult sel =
-            radix_select_range(n_cand, keep, FloatKeys{Sb}, hist, bcast, skmin, skmax);
-        const Segment sg = warp_segment(n_cand);
-        const int eqb = eq_before_segment(Sb, sg, sel, warp_sums, &total_s);
-        const int lane = threadIdx.x & 31;
-        const uint32_t lt = (1u << lane) - 1u;
-        if constexpr (PER <= 16) {
-            // membership ballots kept in registers for the emitting pass (a
-            // warp segment is at most PER x 32 candidates: N <= PER blockDim)
-            uint32_t masks[PER];
-            const int mine = walk_topk_masks_by<PER>(sg, sel, eqb, FloatKeys{Sb}, masks);
-            int pos = warp_exclusive_scan(mine, warp_sums, &total_s);
+        const SelectResult sel = radix_select_range(T * PER, keep, SlotKeys<T, PER>{A2.a, n_cand},
+                                                    hist, bcast, skmin, skmax);
+        const int eqb = ties_before(A2, i0, n_cand, sel, warp_sums, &total_s);
+        const uint32_t mem = members(A2, i0, n_cand, sel, eqb);
+        int pos = block_exclusive_scan(__popc(mem), warp_sums, &total_s);
 #pragma unroll
-            for (int st = 0; st < PER; ++st) {
-                const uint32_t m = masks[st];
-                if ((m >> lane) & 1u) out[pos + __popc(m & lt)] = sg.lo + 32 * st + lane;
-                pos += __popc(m);
-            }
-        } else {
-            // longest prompts: no registers to spare, the keys are walked twice
-            int mine = 0;
-            walk_topk(Sb, sg, sel, eqb, [&](int, bool, bool in) { mine += in; });
-            int pos = warp_exclusive_scan(warp_sum(mine), warp_sums, &total_s);
-            walk_topk(Sb, sg, sel, eqb, [&](int i, bool, bool in) {
-                const uint32_t ball = __ballot_sync(0xffffffffu, in);
-                if (in) out[pos + __popc(ball & lt)] = i;
-                pos += __popc(ball);
-            });
-        }
+        for (int k = 0; k < PER; ++k)
+            if ((mem >> k) & 1u) out[pos++] = i0 + k;
         if (threadIdx.x == 0 && total_s != keep && a.err) atomicCAS(a.err, 0, 2);
     }
     for (int w = threadIdx.x; w < win; w += blockDim.x) out[keep + w] = N - W + w;
@@ -323,7 +463,7 @@ __global__ void __launch_bounds__(T, 1024 / T)
 calibrate_select_kernel(Shape s, Calib c, CalibArgs a)
 {
     const int u = blockIdx.x;
-    calibrate_unit<PER>(s, c, a, u, a.lambda + u, a.idx[u / s.hkv]);
+    calibrate_unit<T, PER>(s, c, a, u, a.lambda + u, a.idx[u / s.hkv]);
 }
 
 // Several hyper-parameter sets over the same B and residuals: CTA (u, v)
@@ -336,19 +476,20 @@ calibrate_sweep_kernel(Shape s, CalibTable t, CalibArgs a)
 {
     const int u = blockIdx.x, v = blockIdx.y;
     float* lam = a.lambda ? a.lambda + (size_t)v * s.units + u : nullptr;
-    calibrate_unit<PER>(s, t.c[v], a, u, lam, a.idx[u / s.hkv] + (size_t)v * a.idx_variant_stride);
+    calibrate_unit<T, PER>(s, t.c[v], a, u, lam,
+                           a.idx[u / s.hkv] + (size_t)v * a.idx_variant_stride);
 }
 
-}  // namespace
-
-size_t calibrate_smem(int N) { return (size_t)2 * N * sizeof(float); }
-
-namespace {
+template <int T, int PER>
+constexpr size_t smem_bytes()
+{
+    return (size_t)2 * T * PER * sizeof(float);
+}
 
 template <int T, int PER>
 cudaError_t launch_select_t(const Shape& s, const Calib& c, const CalibArgs& a, cudaStream_t st)
 {
-    const size_t sm = calibrate_smem(s.N);
+    constexpr size_t sm = smem_bytes<T, PER>();
     cudaError_t e = cudaFuncSetAttribute(calibrate_select_kernel<T, PER>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
@@ -360,7 +501,7 @@ template <int T, int PER>
 cudaError_t launch_sweep_t(const Shape& s, const CalibTable& t, int variants, const CalibArgs& a,
                            cudaStream_t st)
 {
-    const size_t sm = calibrate_smem(s.N);
+    constexpr size_t sm = smem_bytes<T, PER>();
     cudaError_t e = cudaFuncSetAttribute(calibrate_sweep_kernel<T, PER>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
@@ -370,12 +511,20 @@ cudaError_t launch_sweep_t(const Shape& s, const CalibTable& t, int variants, co
 
 }  // namespace
 
+size_t calibrate_smem(int N)
+{
+    if (N <= kSmallPrompt) return smem_bytes<256, kSmallPrompt / 256>();
+    if (N <= kMidPrompt) return smem_bytes<1024, kMidPrompt / 1024>();
+    return smem_bytes<1024, kMaxPrompt / 1024>();
+}
+
 cudaError_t launch_calibrate_select(const Shape& s, const Calib& c, const CalibArgs& a,
                                     cudaStream_t st)
 {
     if (s.N <= kSmallPrompt) return launch_select_t<256, kSmallPrompt / 256>(s, c, a, st);
     if (s.N <= kMidPrompt) return launch_select_t<1024, kMidPrompt / 1024>(s, c, a, st);
-    return launch_select_t<1024, kMaxPer>(s, c, a, st);
+    if (s.N <= kMaxPrompt) return launch_select_t<1024, kMaxPrompt / 1024>(s, c, a, st);
+    return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_calibrate_sweep(const Shape& s, const CalibTable& t, int variants,
@@ -383,7 +532,8 @@ cudaError_t launch_calibrate_sweep(const Shape& s, const CalibTable& t, int vari
 {
     if (s.N <= kSmallPrompt) return launch_sweep_t<256, kSmallPrompt / 256>(s, t, variants, a, st);
     if (s.N <= kMidPrompt) return launch_sweep_t<1024, kMidPrompt / 1024>(s, t, variants, a, st);
-    return launch_sweep_t<1024, kMaxPer>(s, t, variants, a, st);
+    if (s.N <= kMaxPrompt) return launch_sweep_t<1024, kMaxPrompt / 1024>(s, t, variants, a, st);
+    return cudaErrorInvalidValue;
 }
 
 }  // namespace bacon

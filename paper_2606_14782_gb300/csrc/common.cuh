@@ -52,6 +52,14 @@ __device__ __forceinline__ float fast_exp2(float x)
     return y;
 }
 
+// max(a, b, c) in one instruction.
+__device__ __forceinline__ float max3f(float a, float b, float c)
+{
+    float d;
+    asm("max.f32 %0, %1, %2, %3;\n" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
 // Order-preserving map of a float to an unsigned key (larger float ->
 // larger key), used by the radix selections, and its inverse.
 __device__ __forceinline__ uint32_t float_key(float f)

@@ -208,6 +208,24 @@ __device__ __forceinline__ void tmem_ld_wait_regs32(float* v)
     tmem_ld_wait_regs16(v + 16);
 }
 
+// 16 lanes x 32 columns starting at taddr (16x64b shape, 16 repeats): thread
+// t receives lane (t >> 2) + 8 (t & 1) of the 16 and, in register c, column
+// 2 c + ((t >> 1) & 1) (every other column).  This is the layout an M = 64
+// accumulator leaves in the first 16 lanes of each 32-lane quarter.
+__device__ __forceinline__ void tmem_ld16x64b_x16(uint32_t taddr, float* v)
+{
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x64b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
 // Store 32 consecutive fp32 columns of this thread's TMEM lane.
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float* v)
 {

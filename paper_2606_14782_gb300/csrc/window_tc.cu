@@ -69,7 +69,8 @@ struct Smem {
 // so every group of 8 token rows reads the same atom.
 struct Plan {
     int q_rows, n_jobs, granules, stages, nbuf_log2, bias_rows, ones_atom;
-    int q_slots;  // 2: the next unit's window rows load while this unit's MMAs run
+    int q_slots;   // 2: the next unit's window rows load while this unit's MMAs run
+    int last_m64;  // pass 1: the last row block holds 64 window rows (an M = 64 job)
 };
 
 constexpr uint32_t kOnesBytes = 128u * 128u;
@@ -285,7 +286,7 @@ __device__ __forceinline__ void produce(const TcArgs& a, const Smem& L, uint8_t*
 // Pass 2: A = K tile (M = 128 tokens), B = window rows (N = n_h per half).
 template <int D, int PASS, int NBUF_LOG2>
 __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* sm, const Bars& b, int stages,
-                      int q_slots, const JobTable& jt, uint32_t ones_stride)
+                      int q_slots, const JobTable& jt, uint32_t ones_stride, int last_m64)
 {
     const Shape& s = a.s;
     const int ntiles = (s.N + kTileTok - 1) / kTileTok;
@@ -322,7 +323,10 @@ __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* s
                 if (!tc::mbar_wait(b.t_empty(buf), (nb & 1) ^ 1, b.abort())) { ok = false; break; }
                 tc::fence_after_sync();
                 const uint32_t d_tmem = tmem + buf * buf_cols;
-                const uint32_t idesc = tc::idesc_bf16(128, jt.n(j));
+                // pass 1's last row block of 64 window rows: an M = 64 job,
+                // which fills the first 16 lanes of each TMEM lane quarter
+                const int m_rows = (PASS == 1 && last_m64 && j == jt.n_jobs - 1) ? 64 : 128;
+                const uint32_t idesc = tc::idesc_bf16(m_rows, jt.n(j));
                 const uint32_t qaddr = sbase + L.q + cur_slot * L.q_slot + jt.row0(j) * 128;
                 if (PASS == 2)  // D = -lse2 / c per row (columns of D), then += K Q^T
                     tc::umma_bf16(d_tmem, tc::sdesc_sw128(sbase + L.ones, ones_stride),
@@ -351,12 +355,60 @@ __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* s
 
 // ------------------------------------------------- epilogue, pass 1 (stats)
 
+// Folds NV more logits of one row into its running (max, sum of 2^(c x -
+// max)), both in the log2 domain.  Masked logits are -inf.
+template <int NV>
+__device__ __forceinline__ void row_stats(const float* v, float c, unsigned long long c2,
+                                          float& m_run, float& z_run)
+{
+    static_assert(NV == 32 || NV == 16, "32 or 16 logits");
+    float mx;
+    if (NV == 32) {
+        // max of 32 by a tree of 3-input maxima
+        float m9[11];
+#pragma unroll
+        for (int i = 0; i < 10; ++i) m9[i] = tc::max3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+        m9[10] = fmaxf(v[30], v[31]);
+        const float mA = tc::max3(m9[0], m9[1], m9[2]);
+        const float mB = tc::max3(m9[3], m9[4], m9[5]);
+        const float mC = tc::max3(m9[6], m9[7], m9[8]);
+        const float mD = fmaxf(m9[9], m9[10]);
+        mx = fmaxf(tc::max3(mA, mB, mC), mD);
+    } else {
+        float m5[5];
+#pragma unroll
+        for (int i = 0; i < 5; ++i) m5[i] = tc::max3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+        mx = fmaxf(tc::max3(m5[0], m5[1], m5[2]), tc::max3(m5[3], m5[4], v[15]));
+    }
+    const float m_new = fmaxf(m_run, mx * c);
+    if (m_new == -INFINITY) return;
+    const unsigned long long nm2 = tc::pack2(-m_new, -m_new);
+    unsigned long long acc[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll
+    for (int j = 0; j < NV; j += 2) {
+        const float2 tt = tc::unpack2(tc::fma2(tc::pack2(v[j], v[j + 1]), c2, nm2));
+        acc[(j >> 1) & 3] = tc::add2(acc[(j >> 1) & 3], tc::pack2(fast_exp2(tt.x), fast_exp2(tt.y)));
+    }
+    const float2 s2 = tc::unpack2(tc::add2(tc::add2(acc[0], acc[1]), tc::add2(acc[2], acc[3])));
+    const float zs = s2.x + s2.y;
+    if (m_new > m_run) {
+        z_run = z_run * fast_exp2(m_run - m_new) + zs;
+        m_run = m_new;
+    } else {
+        z_run += zs;
+    }
+}
+
 // Thread = one window row (TMEM lane) x one 32-token quarter (its group) of
 // every job; running (max, sum of 2^x) per row block, merged across the
-// groups at the end of each chunk.
+// groups at the end of each chunk.  With last_m64 the last row block is an
+// M = 64 job: its 64 rows sit in the first 16 lanes of each lane quarter,
+// and a thread reads one of them and every other token of its 32 (16x64b
+// shape), so the two threads holding a row combine their statistics before
+// the merge.
 template <int D>
 __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, uint8_t* sm,
-                                               const Bars& b, int q_rows)
+                                               const Bars& b, int q_rows, int last_m64)
 {
     const Shape& s = a.s;
     const int ntiles = (s.N + kTileTok - 1) / kTileTok;
@@ -366,6 +418,10 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
     const uint32_t tmem = tc::ld_shared(b.tmem_slot());
     float2* xchg = reinterpret_cast<float2*>(sm + L.xchg);  // [group][rb][128]
     const int nrb = (q_rows + 127) / 128;
+    const int nfull = last_m64 ? nrb - 1 : nrb;  // 128-row blocks
+    // window row of this thread in the half block, and its tokens 2 c + odd
+    const int row_h = nfull * 128 + quarter * 16 + (lane >> 2) + 8 * (lane & 1);
+    const int odd = (lane >> 1) & 1;
     const float c = kLog2e * rsqrtf((float)D);
     const unsigned long long c2 = tc::pack2(c, c);
     int c0, c1;
@@ -374,22 +430,24 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
     bool ok = true;
     for (int g = c0; g < c1 && ok; ++g) {
         const int u = g / a.chunks, ci = g - u * a.chunks;
+        // running statistics per 128-row block, and of the half block
         float m_run[4], z_run[4];
         int vis[4];
 #pragma unroll
         for (int rb = 0; rb < 4; ++rb) {
             m_run[rb] = -INFINITY;
             z_run[rb] = 0.f;
-            const int r = rb * 128 + quarter * 32 + lane;
-            vis[rb] = s.N - s.W + (r % s.W);
+            vis[rb] = s.N - s.W + ((rb * 128 + quarter * 32 + lane) % s.W);
         }
+        float m_h = -INFINITY, z_h = 0.f;
+        const int vis_h = s.N - s.W + (row_h % s.W);
         const int t1 = min(ntiles, (ci + 1) * kTilesPerChunk);
         for (int t = ci * kTilesPerChunk; t < t1 && ok; ++t) {
             const int tok0 = t * kTileTok + group * 32;
             const bool need_mask = tok0 + 31 > s.N - s.W;
 #pragma unroll
             for (int rb = 0; rb < 4; ++rb) {
-                if (rb >= nrb) break;
+                if (rb >= nfull) break;
                 const int buf = job & 3, nb = job >> 2;
                 ++job;
                 if (!tc::mbar_wait(b.t_full(buf), nb & 1, b.abort())) { ok = false; break; }
@@ -405,36 +463,37 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
                     for (int j = 0; j < 32; ++j)
                         if (tok0 + j > vis[rb]) v[j] = -INFINITY;
                 }
-                // max of 32 by a tree of 3-input maxima
-                float m9[11];
+                row_stats<32>(v, c, c2, m_run[rb], z_run[rb]);
+            }
+            if (last_m64 && ok) {
+                const int buf = job & 3, nb = job >> 2;
+                ++job;
+                if (!tc::mbar_wait(b.t_full(buf), nb & 1, b.abort())) { ok = false; break; }
+                tc::fence_after_sync();
+                float v[16];
+                tc::tmem_ld16x64b_x16(tmem + ((uint32_t)(quarter * 32) << 16) + buf * 128 + group * 32, v);
+                tc::tmem_ld_wait_regs16(v);
+                tc::fence_before_sync();
+                __syncwarp();
+                if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
+                if (need_mask) {
 #pragma unroll
-                for (int i = 0; i < 10; ++i) m9[i] = tc::max3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
-                m9[10] = fmaxf(v[30], v[31]);
-                const float mA = tc::max3(m9[0], m9[1], m9[2]);
-                const float mB = tc::max3(m9[3], m9[4], m9[5]);
-                const float mC = tc::max3(m9[6], m9[7], m9[8]);
-                const float mD = fmaxf(m9[9], m9[10]);
-                const float m_new = fmaxf(m_run[rb], fmaxf(tc::max3(mA, mB, mC), mD) * c);
-                if (m_new != -INFINITY) {
-                    const unsigned long long nm2 = tc::pack2(-m_new, -m_new);
-                    unsigned long long acc[4] = {0ull, 0ull, 0ull, 0ull};
-#pragma unroll
-                    for (int j = 0; j < 32; j += 2) {
-                        const float2 tt = tc::unpack2(tc::fma2(tc::pack2(v[j], v[j + 1]), c2, nm2));
-                        acc[(j >> 1) & 3] = tc::add2(acc[(j >> 1) & 3], tc::pack2(fast_exp2(tt.x), fast_exp2(tt.y)));
-                    }
-                    const float2 s2 = tc::unpack2(tc::add2(tc::add2(acc[0], acc[1]), tc::add2(acc[2], acc[3])));
-                    const float zs = s2.x + s2.y;
-                    if (m_new > m_run[rb]) {
-                        z_run[rb] = z_run[rb] * fast_exp2(m_run[rb] - m_new) + zs;
-                        m_run[rb] = m_new;
-                    } else {
-                        z_run[rb] += zs;
-                    }
+                    for (int j = 0; j < 16; ++j)
+                        if (tok0 + 2 * j + odd > vis_h) v[j] = -INFINITY;
                 }
+                row_stats<16>(v, c, c2, m_h, z_h);
             }
         }
         if (!ok) break;
+        if (last_m64) {
+            // the half block: the two threads of a row (lanes l and l ^ 2)
+            // hold its even and odd tokens; combine them
+            const float mo = __shfl_xor_sync(0xffffffffu, m_h, 2);
+            const float zo = __shfl_xor_sync(0xffffffffu, z_h, 2);
+            const float M = fmaxf(m_h, mo);
+            if (M != -INFINITY) z_h = z_h * fast_exp2(m_h - M) + zo * fast_exp2(mo - M);
+            m_h = M;
+        }
         // merge the groups' statistics of each row and publish the chunk's
         // partial: group n mod 4 of this CTA's n-th chunk waits until the
         // other three groups of its lane quarter have left their (max, sum)
@@ -444,7 +503,7 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
         // is unambiguous only once the barrier's previous phase has
         // completed, and the merging group's x_full wait could otherwise pass
         // on the previous chunk's phase while a slower group is a chunk
-        // behind.
+        // behind.  (A lane holds the same row in every group.)
         const int merger = nch & 3;
         const uint32_t ph = (uint32_t)nch & 1u;
         ++nch;
@@ -456,7 +515,9 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
 #pragma unroll
             for (int rb = 0; rb < 4; ++rb) {
                 if (rb >= nrb) break;
-                xchg[(group * 4 + rb) * 128 + quarter * 32 + lane] = make_float2(m_run[rb], z_run[rb]);
+                const bool h = last_m64 && rb == nfull;
+                xchg[(group * 4 + rb) * 128 + quarter * 32 + lane] =
+                    h ? make_float2(m_h, z_h) : make_float2(m_run[rb], z_run[rb]);
             }
             __syncwarp();
             if (lane == 0) tc::mbar_arrive(b.x_full(0, quarter));
@@ -469,10 +530,12 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
 #pragma unroll
             for (int rb = 0; rb < 4; ++rb) {
                 if (rb >= nrb) break;
+                const bool h = last_m64 && rb == nfull;
                 float2 mz[kGroups];
 #pragma unroll
                 for (int gg = 0; gg < kGroups; ++gg)
-                    mz[gg] = gg == group ? make_float2(m_run[rb], z_run[rb]) : vx[(gg * 4 + rb) * 128];
+                    mz[gg] = gg == group ? (h ? make_float2(m_h, z_h) : make_float2(m_run[rb], z_run[rb]))
+                                         : vx[(gg * 4 + rb) * 128];
                 float M = -INFINITY;
 #pragma unroll
                 for (int gg = 0; gg < kGroups; ++gg) M = fmaxf(M, mz[gg].x);
@@ -484,8 +547,9 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
                         Z = gg == 0 ? zz : Z + zz;
                     }
                 }
-                const int r = rb * 128 + quarter * 32 + lane;
-                if (r < s.rows) a.partial[((size_t)u * a.chunks + ci) * s.rows + r] = make_float2(M, Z);
+                const int r = h ? row_h : rb * 128 + quarter * 32 + lane;
+                if ((!h || (lane & 2) == 0) && r < s.rows)
+                    a.partial[((size_t)u * a.chunks + ci) * s.rows + r] = make_float2(M, Z);
             }
             __syncwarp();
             if (lane == 0) tc::mbar_arrive(b.x_empty(0, quarter));
@@ -806,13 +870,13 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, Plan p
         if (tc::elect_one()) {
             const uint32_t ones_stride = pl.ones_atom ? 0u : 1024u;
             if (pl.nbuf_log2 == 1)
-                issue<D, PASS, 1>(a, L, sm, b, pl.stages, pl.q_slots, jt, ones_stride);
+                issue<D, PASS, 1>(a, L, sm, b, pl.stages, pl.q_slots, jt, ones_stride, pl.last_m64);
             else
-                issue<D, PASS, 2>(a, L, sm, b, pl.stages, pl.q_slots, jt, ones_stride);
+                issue<D, PASS, 2>(a, L, sm, b, pl.stages, pl.q_slots, jt, ones_stride, pl.last_m64);
         }
     } else {
         if (PASS == 1)
-            epilogue_stats<D>(a, L, sm, b, pl.q_rows);
+            epilogue_stats<D>(a, L, sm, b, pl.q_rows, pl.last_m64);
         else if (a.s.W % 16 == 0 && pl.nbuf_log2 == 1)
             epilogue_scores<D, true, 1>(a, L, sm, b, jt);
         else if (a.s.W % 16 == 0)
@@ -857,6 +921,7 @@ cudaError_t launch_impl(const TcArgs& a, cudaStream_t st)
     // more efficient MMA shape) when shared memory allows, else up to 128.
     Plan pl;
     pl.q_rows = (rows + kQBox - 1) / kQBox * kQBox;
+    pl.last_m64 = (PASS == 1 && pl.q_rows % 128 == 64) ? 1 : 0;
     const int granules = (rows + 15) / 16;
     Smem L;
     bool fits = false;

@@ -74,7 +74,7 @@ def test_missing_arrival_times_out_and_the_context_recovers():
 
 
 NOALLOC_CHILD = textwrap.dedent("""
-    import math, sys, time
+    import os, sys, time
     sys.path.insert(0, {root!r})
     import torch
     from paper_2606_14782_gb300 import bacon, build, workloads
@@ -97,6 +97,7 @@ NOALLOC_CHILD = textwrap.dedent("""
 
     t0 = time.time()
     rc, out = call()                    # BACON_FAULT is set: this call's pass 1 loses a load
+    os.environ.pop("BACON_FAULT")       # (the reference context below must not fault)
     print("RC", rc)
     print("SECONDS", round(time.time() - t0, 2))
     print("ALLNAN", int(all(bool(torch.isnan(t).all()) for t in out)))

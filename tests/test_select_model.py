@@ -180,3 +180,90 @@ def test_float_key_orders_like_floats():
     ks = [float_key(x) for x in xs]
     assert ks == sorted(ks)
     assert float_key(-0.0) < float_key(0.0)
+
+
+# ------------------------------------------------ calibration kernel's runs
+
+def slot_major(T, PER):
+    """Storage index of each position in the calibration kernel's
+    shared-memory arrays (thread t owns positions t PER .. t PER + PER - 1;
+    slot k of thread t is stored at k T + t), and its inverse."""
+    at = lambda i: (i % PER) * T + i // PER
+    pos = lambda s: (s % T) * PER + s // T
+    return at, pos
+
+
+def members_by_runs(keys, sel, T, PER):
+    """Membership as the calibration kernel decides it: every thread walks
+    its own run in position order; its tie rank starts from the keys equal
+    to tau in the runs of lower threads (an exclusive scan in thread order),
+    and the members are written at the scan of the per-thread member counts."""
+    tau, need, count_eq = sel
+    n = len(keys)
+    eq_counts = [sum(1 for i in range(t * PER, min(n, t * PER + PER)) if keys[i] == tau)
+                 for t in range(T)]
+    eq_before = [0] * T
+    for t in range(1, T):
+        eq_before[t] = eq_before[t - 1] + eq_counts[t - 1]
+    masks = []
+    for t in range(T):
+        rank = eq_before[t] if need != count_eq else 0
+        m = []
+        for i in range(t * PER, min(n, t * PER + PER)):
+            eq = keys[i] == tau
+            if keys[i] > tau or (eq and (need == count_eq or rank < need)):
+                m.append(i)
+            rank += eq
+        masks.append(m)
+    out = [None] * sum(len(m) for m in masks)
+    pos = 0
+    for m in masks:              # exclusive scan of the member counts
+        for j, i in enumerate(m):
+            out[pos + j] = i
+        pos += len(m)
+    return out
+
+
+@pytest.mark.parametrize("T,PER", [(256, 8), (1024, 16)])
+def test_run_membership_matches_stable_sort(T, PER):
+    for vals, k in cases():
+        if len(vals) > T * PER:
+            continue
+        keys = [float_key(v) for v in vals]
+        # the radix select walks storage indices: the key multiset is the same
+        at, pos = slot_major(T, PER)
+        stored = [None] * (T * PER)
+        for i, key in enumerate(keys):
+            stored[at(i)] = key
+        walked = [stored[s] for s in range(T * PER) if pos(s) < len(keys)]
+        assert sorted(walked) == sorted(keys)
+        sel = radix_select(walked, k)
+        assert members_by_runs(keys, sel, T, PER) == reference(vals, k), (len(vals), k)
+
+
+@pytest.mark.parametrize("T,PER", [(256, 8), (1024, 16), (1024, 24)])
+def test_slot_major_layout_is_a_conflict_free_bijection(T, PER):
+    at, pos = slot_major(T, PER)
+    assert sorted(at(i) for i in range(T * PER)) == list(range(T * PER))
+    assert all(pos(at(i)) == i for i in range(T * PER))
+    # a warp's threads reading their own position plus one offset d touch
+    # 32 consecutive words: 32 distinct banks
+    for w in range(0, T, 32):
+        for d in (-3, -1, 0, 1, 5, PER - 1, PER + 2):
+            words = [at(t * PER + d) for t in range(w, w + 32)
+                     if 0 <= t * PER + d < T * PER]
+            if len(words) == 32:
+                assert len({x % 32 for x in words}) == 32, (w, d)
+
+
+def test_run_membership_without_the_tie_scan_is_caught():
+    """Ranking ties inside each run only (no scan over lower threads) keeps
+    too many equal keys: the comparison above would fail."""
+    vals = [1.0] * 64
+    keys = [float_key(v) for v in vals]
+    sel = radix_select(keys, 10)
+    tau, need, count_eq = sel
+    per_run_only = [i for t in range(8) for j, i in enumerate(range(t * 8, t * 8 + 8))
+                    if keys[i] > tau or j < need]
+    assert per_run_only != reference(vals, 10)
+    assert members_by_runs(keys, sel, 8, 8) == reference(vals, 10)
