@@ -23,7 +23,7 @@ __global__ void __launch_bounds__(kThreads)
 adaptive_select_kernel(Shape s, int keep_window, AdaptArgs a)
 {
     extern __shared__ uint8_t taken[];  // [Hkv][n_cand]
-    __shared__ int hist[kSelHist];
+    __shared__ __align__(16) int hist[kSelHist];
     __shared__ int bcast[8];
     __shared__ int warp_sums[32];
     __shared__ int total_s;

@@ -237,9 +237,9 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
                                                int u, float* lam_out, int32_t* idx_pair)
 {
     extern __shared__ __align__(16) float sm[];
-    const Slots<T, PER> A1{sm};            // B (pooling), then E (coherence)
+    const Slots<T, PER> A1{sm};            // B (pooling), then E (coherence), then V
     const Slots<T, PER> A2{sm + T * PER};  // pooled backbone B~, then the final score S
-    __shared__ int hist[kSelHist];
+    __shared__ __align__(16) int hist[kSelHist];
     __shared__ int bcast[8];
     __shared__ int warp_sums[32];
     __shared__ float red[4 * 33];
@@ -345,6 +345,7 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
         // window sum sliding along the run
         if (c.use_L) {
             const int r = c.r;
+            const float inv_full = 1.f / (float)(2 * r + 1);  // windows away from the ends
             int lo = max(0, i0 - r), hi = min(N - 1, i0 + r);
             float sum = 0.f;
             for (int j = lo; j <= hi; ++j) sum += A1[j];
@@ -355,7 +356,8 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
                     // the window sum of non-negative values: rounding in the
                     // slide can leave ~1e-9 below zero after a large value
                     // leaves the window, so it is clamped
-                    v[k] += fmaxf(sum, 0.f) / (float)(hi - lo + 1);
+                    const int cnt = hi - lo + 1;
+                    v[k] += fmaxf(sum, 0.f) * (cnt == 2 * r + 1 ? inv_full : 1.f / (float)cnt);
                     // the window of i + 1: drop i - r, add i + 1 + r
                     if (i - r >= 0) sum -= A1[i - r];
                     if (i + 1 + r <= N - 1) sum += A1[i + 1 + r];
@@ -371,6 +373,11 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
             if (i0 + k < n_cand) vsum += v[k];
         }
         if (a.V) store_run<PER>(a.V + (size_t)u * N, i0, N, v);
+        // V moves to the E array (own slots) for the rest of the unit: it
+        // is read only by its own thread from here on
+        __syncthreads();  // every coherence read of A1 is done
+#pragma unroll
+        for (int k = 0; k < PER; ++k) A1.own(k) = v[k];
         if (a.Bp) {
 #pragma unroll
             for (int k = 0; k < PER; ++k) x[k] = A2.own(k);
@@ -383,20 +390,22 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
         const int M = (int)(Ml < n_cand ? Ml : n_cand);
         float lam = 0.f;
         if (M > 0) {
+            // (the candidates' V sum rides on the selection's first reduction)
+            float vtot = 0.f;
             const SelectResult sel = radix_select_range(T * PER, M, SlotKeys<T, PER>{A2.a, n_cand},
-                                                        hist, bcast, kmin, kmax);
+                                                        hist, bcast, kmin, kmax, vsum, &vtot);
             const int eqb = ties_before(A2, i0, n_cand, sel, warp_sums, &total_s);
             const uint32_t mem = members(A2, i0, n_cand, sel, eqb);
             // moments about fixed shifts in one walk: B~ about its M-th value,
             // V about its mean over the candidates (both near the members'
             // means, so the fp32 differences keep their precision)
             const float pb = key_float(sel.tau);
-            const float pv = block_sum(vsum, red) / (float)n_cand;
+            const float pv = vtot / (float)n_cand;
             float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
             for (int k = 0; k < PER; ++k) {
                 if ((mem >> k) & 1u) {
-                    const float db = A2.own(k) - pb, dv = v[k] - pv;
+                    const float db = A2.own(k) - pb, dv = A1.own(k) - pv;
                     acc.x += db;
                     acc.y = fmaf(db, db, acc.y);
                     acc.z += dv;
@@ -416,7 +425,7 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
         for (int k = 0; k < PER; ++k) {
             float sv = 0.f;
             if (i0 + k < n_cand) {
-                sv = fmaf(lam, v[k], A2.own(k));
+                sv = fmaf(lam, A1.own(k), A2.own(k));
                 skmin = min(skmin, float_key(sv));
                 skmax = max(skmax, float_key(sv));
             }

@@ -28,49 +28,70 @@ struct SelectResult {
     __device__ __forceinline__ bool all_ties_in() const { return need == count_eq; }
 };
 
-// Histogram bins of one select pass; the caller's shared array `hist` holds
-// kSelHist ints: the bins, 32 warp totals, a counter and a buffer of up to
-// kSelCap keys.
+// Histogram bins of one select pass; the caller's shared array `hist` (16-
+// byte aligned) holds kSelHist ints: two bin buffers (passes alternate, so a
+// pass zeroes the next one's bins while it counts), 128 ints for the
+// reductions and the buffer counter, and a buffer of up to kSelCap keys.
 constexpr int kSelBits = 11;
 constexpr int kSelBins = 1 << kSelBits;
 constexpr int kSelCap = 2048;
-constexpr int kSelHist = kSelBins + 64 + kSelCap;
+constexpr int kSelHist = 2 * kSelBins + 128 + kSelCap;
 
 // k-th best key over the included elements of [0, n) (1 <= k <= their
 // count).  First the range [kmin, kmax] of the included keys, then passes
 // over it: each pass histograms the keys of the current range into
 // kSelBins bins of 2^shift keys (plain shared-memory adds: the bins follow
-// the data's own range, so few keys share one), takes the bin where the
-// count from the top reaches k, and narrows the range to it, until a bin is
-// one key, or until it holds at most 32 keys, which one warp then sorts.
-// At most three passes for 32-bit keys.  Every thread returns the
-// same result; blockDim.x must be a power of two from 64 to 1024.
-// kmin / kmax: this thread's share of the key range (the callers that know
-// it from an earlier pass over the keys pass it in; see radix_select_by).
+// the data's own range, so few keys share one), one warp finds the bin
+// where the count from the top reaches k, and the range narrows to it,
+// until a bin is one key, or until it holds at most 32 keys, which one warp
+// then sorts.  At most three passes for 32-bit keys, two block-wide
+// barriers each.  Every thread returns the same result; blockDim.x must be
+// a multiple of 32 from 64 to 1024.  kmin / kmax: this thread's share of the
+// key range (the callers know it from an earlier pass over the keys).  With
+// fsum, the block-wide sum of every thread's fval is reduced on the same
+// barriers and written to *fsum for every thread.
 template <typename KeyFn>
 __device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist, int* bcast,
-                                           uint32_t kmin, uint32_t kmax)
+                                           uint32_t kmin, uint32_t kmax, float fval = 0.f,
+                                           float* fsum = nullptr)
 {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nwarps = (int)(blockDim.x >> 5);
+    int* const bins0 = hist;
+    int* const red = hist + 2 * kSelBins;  // [0, 32) min, [32, 64) max, [64, 96) sums, [96] counter
+    int* const bufcnt = red + 96;
+    uint32_t* const buf = reinterpret_cast<uint32_t*>(hist + 2 * kSelBins + 128);
     kmin = __reduce_min_sync(0xffffffffu, kmin);
     kmax = __reduce_max_sync(0xffffffffu, kmax);
-    if (lane == 0) {
-        hist[warp] = (int)kmin;
-        hist[32 + warp] = (int)kmax;
+    if (fsum) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) fval += __shfl_xor_sync(0xffffffffu, fval, o);
     }
+    if (lane == 0) {
+        red[warp] = (int)kmin;
+        red[32 + warp] = (int)kmax;
+        reinterpret_cast<float*>(red)[64 + warp] = fval;
+    }
+    for (int b = threadIdx.x; b < kSelBins; b += blockDim.x) bins0[b] = 0;
     __syncthreads();
     if (warp == 0) {
         // only the first nwarps entries were written: the other lanes take
         // the neutral element of each reduction
-        const bool held = lane < (int)(blockDim.x >> 5);
-        const uint32_t a = __reduce_min_sync(0xffffffffu, held ? (uint32_t)hist[lane] : 0xffffffffu);
-        const uint32_t b = __reduce_max_sync(0xffffffffu, held ? (uint32_t)hist[32 + lane] : 0u);
+        const bool held = lane < nwarps;
+        const uint32_t a = __reduce_min_sync(0xffffffffu, held ? (uint32_t)red[lane] : 0xffffffffu);
+        const uint32_t b = __reduce_max_sync(0xffffffffu, held ? (uint32_t)red[32 + lane] : 0u);
+        float f = held ? reinterpret_cast<const float*>(red)[64 + lane] : 0.f;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) f += __shfl_xor_sync(0xffffffffu, f, o);
         if (lane == 0) {
             bcast[0] = (int)a;
             bcast[1] = (int)b;
+            reinterpret_cast<float*>(bcast)[5] = f;
+            *bufcnt = 0;
         }
     }
     __syncthreads();
+    if (fsum) *fsum = reinterpret_cast<const float*>(bcast)[5];
     uint32_t lo = (uint32_t)bcast[0];
     const uint64_t span = (uint64_t)(uint32_t)bcast[1] - lo + 1u;
     int shift = 0;
@@ -79,19 +100,18 @@ __device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist
     int remaining = k;
     // Once the current range holds at most kSelCap keys, the next pass also
     // copies them into the buffer and the passes after it read only that.
-    int* bufcnt = hist + kSelBins + 32;
-    uint32_t* buf = reinterpret_cast<uint32_t*>(hist + kSelBins + 64);
     int in_range = -1, nbuf = -1;  // unknown / not compacted
-    __syncthreads();
-    while (true) {
-        for (int b = threadIdx.x; b < kSelBins; b += blockDim.x) hist[b] = 0;
+    for (int pass = 0;; ++pass) {
+        int* const h = hist + (pass & 1) * kSelBins;          // zeroed
+        int* const hn = hist + ((pass + 1) & 1) * kSelBins;   // the next pass's
         const bool collect = nbuf < 0 && in_range >= 0 && in_range <= kSelCap;
-        if (threadIdx.x == 0) *bufcnt = 0;
-        __syncthreads();
+        // the bins of the pass before this one were last read before the
+        // barrier that ended it: free to zero for the next pass
+        for (int b = threadIdx.x; b < kSelBins; b += blockDim.x) hn[b] = 0;
         if (nbuf >= 0) {
             for (int i = threadIdx.x; i < nbuf; i += blockDim.x) {
                 const uint32_t key = buf[i];
-                if (key >= lo && (uint64_t)(key - lo) < width) atomicAdd(&hist[(key - lo) >> shift], 1);
+                if (key >= lo && (uint64_t)(key - lo) < width) atomicAdd(&h[(key - lo) >> shift], 1);
             }
         } else {
             for (int i0 = threadIdx.x; i0 < n; i0 += 4 * blockDim.x) {
@@ -100,80 +120,68 @@ __device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist
                     const int i = i0 + q * (int)blockDim.x;
                     uint32_t key = 0u;
                     if (i < n && key_of(i, key) && key >= lo && (uint64_t)(key - lo) < width) {
-                        atomicAdd(&hist[(key - lo) >> shift], 1);
+                        atomicAdd(&h[(key - lo) >> shift], 1);
                         if (collect) buf[atomicAdd(bufcnt, 1)] = key;
                     }
                 }
             }
         }
         __syncthreads();
-        if (collect) nbuf = *bufcnt;
-        // bins from the top: warp w holds the w-th slice of bpw bins and its
-        // lane l the bpl bins just below the top l bpl of that slice; warp
-        // totals first, then the boundary warp's lanes, then the lane's bins
-        const int nwarps = (int)(blockDim.x >> 5);
-        const int bpw = kSelBins / nwarps, bpl = bpw / 32;
-        const int ltop = bpw * (warp + 1) - 1 - bpl * lane;  // this lane's highest bin
-        int mine = 0;
-        for (int q = 0; q < bpl; ++q) mine += hist[ltop - q];
-        int incl = mine;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, incl, o);
-            if (lane >= o) incl += y;
-        }
-        if (lane == 31) hist[kSelBins + warp] = incl;  // warp total
-        __syncthreads();
         if (warp == 0) {
-            // warps from the top: above[w] = totals of warps w + 1 .. nwarps - 1
-            const int tot = lane < nwarps ? hist[kSelBins + nwarps - 1 - lane] : 0;
-            int cum = tot;
+            // lane l owns bins [64 l, 64 l + 64); counts from the top are
+            // suffix sums over the lanes (16-byte reads in a rotated order)
+            const int4* h4 = reinterpret_cast<const int4*>(h) + 16 * lane;
+            int mine = 0;
+#pragma unroll
+            for (int q = 0; q < 16; ++q) {
+                const int4 v = h4[(q + lane) & 15];
+                mine += v.x + v.y + v.z + v.w;
+            }
+            int incl = mine;
 #pragma unroll
             for (int o = 1; o < 32; o <<= 1) {
-                const int y = __shfl_up_sync(0xffffffffu, cum, o);
-                if (lane >= o) cum += y;
+                const int y = __shfl_down_sync(0xffffffffu, incl, o);
+                if (lane + o < 32) incl += y;
             }
-            const uint32_t hit = __ballot_sync(0xffffffffu, cum >= remaining);
-            const int first = __ffs(hit) - 1;  // the boundary warp is nwarps - 1 - first
-            const int above = __shfl_sync(0xffffffffu, cum - tot, first);
-            if (lane == 0) {
-                bcast[2] = nwarps - 1 - first;
-                bcast[3] = above;
+            // the boundary lane: the highest one whose count from the top
+            // reaches `remaining`
+            const uint32_t hit = __ballot_sync(0xffffffffu, incl >= remaining);
+            const int lb = hit ? 31 - __clz(hit) : 0;
+            const int above = __shfl_sync(0xffffffffu, incl - mine, lb);
+            // its 64 bins: two per lane, suffix sums again
+            const int b0 = 64 * lb + 2 * lane;
+            const int c0 = h[b0], c1 = h[b0 + 1];
+            const int pair = c0 + c1;
+            int inc2 = pair;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_down_sync(0xffffffffu, inc2, o);
+                if (lane + o < 32) inc2 += y;
+            }
+            const uint32_t hit2 = __ballot_sync(0xffffffffu, above + inc2 >= remaining);
+            const int l2 = hit2 ? 31 - __clz(hit2) : 0;
+            if (lane == l2) {
+                const int before = above + inc2 - pair;  // bins above this pair
+                const bool top = before + c1 >= remaining;
+                bcast[0] = top ? b0 + 1 : b0;
+                bcast[1] = top ? remaining - before : remaining - before - c1;
+                bcast[4] = top ? c1 : c0;
+                bcast[3] = collect ? *bufcnt : -1;
+                *bufcnt = 0;
             }
         }
         __syncthreads();
-        if (warp == bcast[2]) {
-            const int rem = remaining - bcast[3];
-            const uint32_t hit = __ballot_sync(0xffffffffu, incl >= rem);
-            const int first = __ffs(hit) - 1;
-            if (lane == first) {
-                int before = incl - mine;  // bins above this lane's
-                for (int q = 0; q < bpl; ++q) {
-                    const int c = hist[ltop - q];
-                    if (before + c >= rem) {
-                        bcast[0] = ltop - q;
-                        bcast[1] = rem - before;
-                        bcast[4] = c;
-                        break;
-                    }
-                    before += c;
-                }
-            }
-        }
-        __syncthreads();
+        if (collect) nbuf = bcast[3];
         lo += (uint32_t)bcast[0] << shift;
         remaining = bcast[1];
         const int in_bin = bcast[4];
         in_range = in_bin;
         width = (uint64_t)1 << shift;
-        __syncthreads();
         if (shift == 0) return {lo, remaining, in_bin};
         if (in_bin <= 32) {
-            // few keys left in the range: gather them (the bins are free
-            // now) and let one warp sort them instead of more passes
-            int* few = hist;
-            if (threadIdx.x == 0) *bufcnt = 0;
-            __syncthreads();
+            // few keys left in the range: gather them (this pass's bins are
+            // free now) and let one warp sort them instead of more passes
+            int* few = h;
             if (nbuf >= 0) {
                 for (int i = threadIdx.x; i < nbuf; i += blockDim.x) {
                     const uint32_t key = buf[i];
@@ -193,11 +201,11 @@ __device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist
                 unsigned long long v =
                     lane < in_bin ? ((1ull << 32) | (uint32_t)few[lane]) : 0ull;
 #pragma unroll
-                for (int k = 2; k <= 32; k <<= 1) {
+                for (int kk = 2; kk <= 32; kk <<= 1) {
 #pragma unroll
-                    for (int j = k >> 1; j > 0; j >>= 1) {
+                    for (int j = kk >> 1; j > 0; j >>= 1) {
                         const unsigned long long o = __shfl_xor_sync(0xffffffffu, v, j);
-                        const bool keep_max = ((lane & k) == 0) == ((lane & j) == 0);
+                        const bool keep_max = ((lane & kk) == 0) == ((lane & j) == 0);
                         v = keep_max ? (v > o ? v : o) : (v < o ? v : o);
                     }
                 }
@@ -210,12 +218,11 @@ __device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist
                     bcast[0] = (int)tau;
                     bcast[1] = remaining - gt;
                     bcast[4] = eq;
+                    *bufcnt = 0;
                 }
             }
             __syncthreads();
-            const SelectResult r = {(uint32_t)bcast[0], bcast[1], bcast[4]};
-            __syncthreads();
-            return r;
+            return {(uint32_t)bcast[0], bcast[1], bcast[4]};
         }
         shift = shift > kSelBits ? shift - kSelBits : 0;
     }

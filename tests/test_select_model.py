@@ -267,3 +267,77 @@ def test_run_membership_without_the_tie_scan_is_caught():
                     if keys[i] > tau or j < need]
     assert per_run_only != reference(vals, 10)
     assert members_by_runs(keys, sel, 8, 8) == reference(vals, 10)
+
+
+# ---------------------------------- boundary search of one histogram pass
+
+def boundary_direct(hist, remaining):
+    """The bin where the count from the top reaches `remaining`: (bin, keys
+    still needed inside it, its count)."""
+    before = 0
+    for b in range(len(hist) - 1, -1, -1):
+        if before + hist[b] >= remaining:
+            return b, remaining - before, hist[b]
+        before += hist[b]
+    raise AssertionError("fewer keys than requested")
+
+
+def boundary_by_warp(hist, remaining):
+    """The single warp's search: lane l owns bins [64 l, 64 l + 64); suffix
+    sums over the lanes find the highest lane whose count from the top
+    reaches `remaining`; its 64 bins, two per lane, go through the same
+    suffix-sum search; the chosen pair's upper bin is taken if it alone
+    completes the count, else the lower one."""
+    assert len(hist) == 2048
+    mine = [sum(hist[64 * l:64 * l + 64]) for l in range(32)]
+    incl = [sum(mine[l:]) for l in range(32)]           # shfl_down suffix scan
+    hit = [incl[l] >= remaining for l in range(32)]
+    lb = max(l for l in range(32) if hit[l])
+    above = incl[lb] - mine[lb]
+    pairs = [(hist[64 * lb + 2 * l], hist[64 * lb + 2 * l + 1]) for l in range(32)]
+    inc2 = [sum(c0 + c1 for c0, c1 in pairs[l:]) for l in range(32)]
+    l2 = max(l for l in range(32) if above + inc2[l] >= remaining)
+    c0, c1 = pairs[l2]
+    before = above + inc2[l2] - (c0 + c1)
+    b0 = 64 * lb + 2 * l2
+    if before + c1 >= remaining:
+        return b0 + 1, remaining - before, c1
+    return b0, remaining - before - c1, c0
+
+
+def test_warp_boundary_search_matches_direct_scan():
+    rng = random.Random(11)
+    for trial in range(400):
+        kind = trial % 4
+        if kind == 0:      # sparse: few occupied bins, long runs of zeros
+            hist = [0] * 2048
+            for _ in range(rng.randint(1, 40)):
+                hist[rng.randrange(2048)] += rng.randint(1, 50)
+        elif kind == 1:    # dense
+            hist = [rng.randint(0, 9) for _ in range(2048)]
+        elif kind == 2:    # one heavy bin
+            hist = [0] * 2048
+            hist[rng.randrange(2048)] = rng.randint(1, 16000)
+        else:              # occupied bins only at a lane's edges
+            hist = [0] * 2048
+            for l in range(32):
+                if rng.random() < 0.5:
+                    hist[64 * l + rng.choice([0, 1, 62, 63])] = rng.randint(1, 5)
+            if not sum(hist):
+                hist[0] = 1
+        total = sum(hist)
+        for remaining in sorted({1, total, max(1, total // 2), rng.randint(1, total)}):
+            assert boundary_by_warp(hist, remaining) == boundary_direct(hist, remaining), (
+                trial, remaining)
+
+
+def test_warp_boundary_search_with_the_wrong_pair_order_is_caught():
+    """Taking the pair's lower bin first (the wrong end of the suffix order)
+    picks a bin below the boundary: the comparison above would fail."""
+    hist = [0] * 2048
+    hist[100], hist[101] = 3, 4        # one pair, upper bin 101 holds 4
+    b, need, cnt = boundary_direct(hist, 2)
+    assert (b, need, cnt) == (101, 2, 4)
+    assert boundary_by_warp(hist, 2) == (101, 2, 4)
+    # lower bin first: 100 would be reported
+    assert b != 100
