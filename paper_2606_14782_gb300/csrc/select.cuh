@@ -114,12 +114,13 @@ __device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist
                 if (key >= lo && (uint64_t)(key - lo) < width) atomicAdd(&h[(key - lo) >> shift], 1);
             }
         } else {
+            const uint32_t last = (uint32_t)(width - 1u);  // width <= 2^32
             for (int i0 = threadIdx.x; i0 < n; i0 += 4 * blockDim.x) {
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
                     const int i = i0 + q * (int)blockDim.x;
                     uint32_t key = 0u;
-                    if (i < n && key_of(i, key) && key >= lo && (uint64_t)(key - lo) < width) {
+                    if (i < n && key_of(i, key) && key >= lo && key - lo <= last) {
                         atomicAdd(&h[(key - lo) >> shift], 1);
                         if (collect) buf[atomicAdd(bufcnt, 1)] = key;
                     }
@@ -188,10 +189,17 @@ __device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist
                     if (key >= lo && (uint64_t)(key - lo) < width) few[atomicAdd(bufcnt, 1)] = (int)key;
                 }
             } else {
-                for (int i = threadIdx.x; i < n; i += blockDim.x) {
-                    uint32_t key = 0u;
-                    if (key_of(i, key) && key >= lo && (uint64_t)(key - lo) < width)
-                        few[atomicAdd(bufcnt, 1)] = (int)key;
+                // four keys per iteration, as in the histogram pass: the
+                // loads of a thread's keys are in flight together
+                const uint32_t last = (uint32_t)(width - 1u);
+                for (int i0 = threadIdx.x; i0 < n; i0 += 4 * blockDim.x) {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const int i = i0 + q * (int)blockDim.x;
+                        uint32_t key = 0u;
+                        if (i < n && key_of(i, key) && key >= lo && key - lo <= last)
+                            few[atomicAdd(bufcnt, 1)] = (int)key;
+                    }
                 }
             }
             __syncthreads();

@@ -355,16 +355,12 @@ __device__ __forceinline__ void issue(const TcArgs& a, const Smem& L, uint8_t* s
 
 // ------------------------------------------------- epilogue, pass 1 (stats)
 
-// Folds NV more logits of one row into its running (max, sum of 2^(c x -
-// max)), both in the log2 domain.  Masked logits are -inf.
+// Maximum of NV logits by a tree of 3-input maxima.
 template <int NV>
-__device__ __forceinline__ void row_stats(const float* v, float c, unsigned long long c2,
-                                          float& m_run, float& z_run)
+__device__ __forceinline__ float max_tree(const float* v)
 {
     static_assert(NV == 32 || NV == 16, "32 or 16 logits");
-    float mx;
     if (NV == 32) {
-        // max of 32 by a tree of 3-input maxima
         float m9[11];
 #pragma unroll
         for (int i = 0; i < 10; ++i) m9[i] = tc::max3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
@@ -373,13 +369,23 @@ __device__ __forceinline__ void row_stats(const float* v, float c, unsigned long
         const float mB = tc::max3(m9[3], m9[4], m9[5]);
         const float mC = tc::max3(m9[6], m9[7], m9[8]);
         const float mD = fmaxf(m9[9], m9[10]);
-        mx = fmaxf(tc::max3(mA, mB, mC), mD);
-    } else {
-        float m5[5];
-#pragma unroll
-        for (int i = 0; i < 5; ++i) m5[i] = tc::max3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
-        mx = fmaxf(tc::max3(m5[0], m5[1], m5[2]), tc::max3(m5[3], m5[4], v[15]));
+        return fmaxf(tc::max3(mA, mB, mC), mD);
     }
+    float m5[5];
+#pragma unroll
+    for (int i = 0; i < 5; ++i) m5[i] = tc::max3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+    return fmaxf(tc::max3(m5[0], m5[1], m5[2]), tc::max3(m5[3], m5[4], v[15]));
+}
+
+// Folds NV more logits of one row, whose maximum is mx, into its running
+// (max, sum of 2^(c x - max)), both in the log2 domain.  Masked logits are
+// -inf.  (Exponentiating against the running maximum and redoing a job only
+// when its sum overflows would save the maximum but costs a data-dependent
+// branch per job, which measured slower than computing it.)
+template <int NV>
+__device__ __forceinline__ void row_stats(const float* v, float mx, float c, unsigned long long c2,
+                                          float& m_run, float& z_run)
+{
     const float m_new = fmaxf(m_run, mx * c);
     if (m_new == -INFINITY) return;
     const unsigned long long nm2 = tc::pack2(-m_new, -m_new);
@@ -430,7 +436,10 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
     bool ok = true;
     for (int g = c0; g < c1 && ok; ++g) {
         const int u = g / a.chunks, ci = g - u * a.chunks;
-        // running statistics per 128-row block, and of the half block
+        // running statistics per 128-row block, and of the half block,
+        // restarted at every chunk: a chunk's partial depends on its own
+        // logits only, whichever CTA and range of chunks processes it (every
+        // launch shape gives the same bits)
         float m_run[4], z_run[4];
         int vis[4];
 #pragma unroll
@@ -452,18 +461,22 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
                 ++job;
                 if (!tc::mbar_wait(b.t_full(buf), nb & 1, b.abort())) { ok = false; break; }
                 tc::fence_after_sync();
-                float v[32];
-                tc::tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + buf * 128 + group * 32, v);
-                tc::tmem_ld_wait_regs32(v);
+                // the load also reduces the 32 logits to their maximum
+                float v[32], mx;
+                tc::tmem_ld32_max(tmem + ((uint32_t)(quarter * 32) << 16) + buf * 128 + group * 32, v,
+                                  mx);
+                tc::tmem_ld_wait_regs32_max(v, mx);
                 tc::fence_before_sync();
                 __syncwarp();
                 if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
                 if (need_mask) {
+                    // tiles that reach into the window: mask, then the tree
 #pragma unroll
                     for (int j = 0; j < 32; ++j)
                         if (tok0 + j > vis[rb]) v[j] = -INFINITY;
+                    mx = max_tree<32>(v);
                 }
-                row_stats<32>(v, c, c2, m_run[rb], z_run[rb]);
+                row_stats<32>(v, mx, c, c2, m_run[rb], z_run[rb]);
             }
             if (last_m64 && ok) {
                 const int buf = job & 3, nb = job >> 2;
@@ -481,7 +494,7 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
                     for (int j = 0; j < 16; ++j)
                         if (tok0 + 2 * j + odd > vis_h) v[j] = -INFINITY;
                 }
-                row_stats<16>(v, c, c2, m_h, z_h);
+                row_stats<16>(v, max_tree<16>(v), c, c2, m_h, z_h);
             }
         }
         if (!ok) break;
@@ -599,20 +612,27 @@ __device__ __forceinline__ void score_slice(float* v, int r0, int tok, const Sco
         }
     }
     int rm = FASTQ ? 0 : r0 % k.W;
+    float q_end[NC / 16];  // FASTQ: the exponentials of the granules' last rows
 #pragma unroll
     for (int j = 0; j < NC; j += 2) {
         const float2 t = tc::unpack2(tc::mul2(tc::pack2(v[j], v[j + 1]), k.c2));
         const float x0 = fast_exp2(t.x), x1 = fast_exp2(t.y);
         bacc[(j >> 1) & 1] = tc::add2(bacc[(j >> 1) & 1], tc::pack2(x0, x1));
         if (FASTQ) {
-            // with W a multiple of 16 only a granule's last row can be a last-position row
-            if ((j & 15) == 14 && ((k.qmask >> ((r0 + j) >> 4)) & 1u)) qacc += x1;
+            if ((j & 15) == 14) q_end[j >> 4] = x1;
         } else {
             if (rm == k.W - 1) qacc += x0;
             rm = rm + 1 == k.W ? 0 : rm + 1;
             if (rm == k.W - 1) qacc += x1;
             rm = rm + 1 == k.W ? 0 : rm + 1;
         }
+    }
+    if (FASTQ) {
+        // with W a multiple of 16 only a granule's last row can be a
+        // last-position row: one mask test per granule, after the loop
+#pragma unroll
+        for (int g = 0; g < NC / 16; ++g)
+            if ((k.qmask >> ((r0 >> 4) + g)) & 1u) qacc += q_end[g];
     }
 }
 
