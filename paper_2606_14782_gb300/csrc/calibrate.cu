@@ -33,11 +33,11 @@ using namespace sel;
 
 // Threads per CTA and positions per thread depend on the prompt length only
 // (so that every call on the same shape reduces in the same order and gives
-// the same bits): 256 threads of 8 positions up to 2048 tokens, where
-// several CTAs share an SM; 1024 threads of 16 positions up to 16384
-// tokens; 1024 threads of 24 above (up to 24576).
-constexpr int kSmallPrompt = 2048;
-constexpr int kMidPrompt = 16384;
+// the same bits), sized so that threads x positions stays close to N (the
+// selections walk every storage slot): 8 positions per thread on 128, 256,
+// 512 or 1024 threads up to 1024, 2048, 4096 or 8192 tokens (several CTAs
+// share an SM below 1024 threads), then 1024 threads of 16 positions up to
+// 16384 tokens and of 24 up to 24576.
 constexpr int kMaxPrompt = 24576;
 
 // Block-wide fp32 sum by a shuffle tree (pairwise, so the rounding error
@@ -518,31 +518,67 @@ cudaError_t launch_sweep_t(const Shape& s, const CalibTable& t, int variants, co
     return cudaGetLastError();
 }
 
+// The launch for a prompt of N tokens: F(T, PER) with the size class above.
+template <typename F>
+cudaError_t by_size(int N, F f)
+{
+    if (N <= 1024) return f.template run<128, 8>();
+    if (N <= 2048) return f.template run<256, 8>();
+    if (N <= 4096) return f.template run<512, 8>();
+    if (N <= 8192) return f.template run<1024, 8>();
+    if (N <= 16384) return f.template run<1024, 16>();
+    if (N <= kMaxPrompt) return f.template run<1024, 24>();
+    return cudaErrorInvalidValue;
+}
+
+struct SmemOf {
+    size_t* out;
+    template <int T, int PER>
+    cudaError_t run() const
+    {
+        *out = smem_bytes<T, PER>();
+        return cudaSuccess;
+    }
+};
+
+struct SelectLaunch {
+    const Shape& s;
+    const Calib& c;
+    const CalibArgs& a;
+    cudaStream_t st;
+    template <int T, int PER>
+    cudaError_t run() const { return launch_select_t<T, PER>(s, c, a, st); }
+};
+
+struct SweepLaunch {
+    const Shape& s;
+    const CalibTable& t;
+    int variants;
+    const CalibArgs& a;
+    cudaStream_t st;
+    template <int T, int PER>
+    cudaError_t run() const { return launch_sweep_t<T, PER>(s, t, variants, a, st); }
+};
+
 }  // namespace
 
 size_t calibrate_smem(int N)
 {
-    if (N <= kSmallPrompt) return smem_bytes<256, kSmallPrompt / 256>();
-    if (N <= kMidPrompt) return smem_bytes<1024, kMidPrompt / 1024>();
-    return smem_bytes<1024, kMaxPrompt / 1024>();
+    size_t bytes = 0;
+    by_size(N, SmemOf{&bytes});
+    return bytes;
 }
 
 cudaError_t launch_calibrate_select(const Shape& s, const Calib& c, const CalibArgs& a,
                                     cudaStream_t st)
 {
-    if (s.N <= kSmallPrompt) return launch_select_t<256, kSmallPrompt / 256>(s, c, a, st);
-    if (s.N <= kMidPrompt) return launch_select_t<1024, kMidPrompt / 1024>(s, c, a, st);
-    if (s.N <= kMaxPrompt) return launch_select_t<1024, kMaxPrompt / 1024>(s, c, a, st);
-    return cudaErrorInvalidValue;
+    return by_size(s.N, SelectLaunch{s, c, a, st});
 }
 
 cudaError_t launch_calibrate_sweep(const Shape& s, const CalibTable& t, int variants,
                                    const CalibArgs& a, cudaStream_t st)
 {
-    if (s.N <= kSmallPrompt) return launch_sweep_t<256, kSmallPrompt / 256>(s, t, variants, a, st);
-    if (s.N <= kMidPrompt) return launch_sweep_t<1024, kMidPrompt / 1024>(s, t, variants, a, st);
-    if (s.N <= kMaxPrompt) return launch_sweep_t<1024, kMaxPrompt / 1024>(s, t, variants, a, st);
-    return cudaErrorInvalidValue;
+    return by_size(s.N, SweepLaunch{s, t, variants, a, st});
 }
 
 }  // namespace bacon

@@ -224,7 +224,7 @@ def members_by_runs(keys, sel, T, PER):
     return out
 
 
-@pytest.mark.parametrize("T,PER", [(256, 8), (1024, 16)])
+@pytest.mark.parametrize("T,PER", [(128, 8), (256, 8), (512, 8), (1024, 8), (1024, 16)])
 def test_run_membership_matches_stable_sort(T, PER):
     for vals, k in cases():
         if len(vals) > T * PER:
@@ -241,7 +241,7 @@ def test_run_membership_matches_stable_sort(T, PER):
         assert members_by_runs(keys, sel, T, PER) == reference(vals, k), (len(vals), k)
 
 
-@pytest.mark.parametrize("T,PER", [(256, 8), (1024, 16), (1024, 24)])
+@pytest.mark.parametrize("T,PER", [(128, 8), (256, 8), (512, 8), (1024, 8), (1024, 16), (1024, 24)])
 def test_slot_major_layout_is_a_conflict_free_bijection(T, PER):
     at, pos = slot_major(T, PER)
     assert sorted(at(i) for i in range(T * PER)) == list(range(T * PER))
