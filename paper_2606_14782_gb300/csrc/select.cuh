@@ -51,7 +51,7 @@ constexpr int kSelHist = 2 * kSelBins + 128 + kSelCap;
 // fsum, the block-wide sum of every thread's fval is reduced on the same
 // barriers and written to *fsum for every thread.
 template <typename KeyFn>
-__device__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist, int* bcast,
+__device__ __noinline__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist, int* bcast,
                                            uint32_t kmin, uint32_t kmax, float fval = 0.f,
                                            float* fsum = nullptr)
 {

@@ -10,7 +10,7 @@ import torch
 
 import oracle
 from paper_2606_14782_gb300 import bacon, build, workloads
-from parity import check_scores, check_selection, record_swaps
+from parity import ATOL, RTOL, check_scores, check_selection, record_swaps
 
 pytestmark = pytest.mark.gpu
 
@@ -66,7 +66,7 @@ def compare(wl, x, budget, gpu, orc, report=None, case=None, path="whole step"):
             e, _ = check_scores(f"{where} {name}", gpu[name][r, l, h], o[okey])
             worst = max(worst, e)
         lam_g, lam_o = float(gpu["lambda"][r, l, h]), o["lambda"]
-        assert abs(lam_g - lam_o) <= 1e-2 * abs(lam_o) + 1e-6, (where, lam_g, lam_o)
+        assert abs(lam_g - lam_o) <= RTOL * abs(lam_o) + ATOL, (where, lam_g, lam_o)
         gi = gpu["idx"][r, l, h]
         swaps += check_selection(gi, o["idx"], o["S"], N, W, budget, keep_window=kw, log=log,
                                  unit=key)

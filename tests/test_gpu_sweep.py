@@ -10,7 +10,7 @@ import pytest
 
 import oracle
 from paper_2606_14782_gb300 import bacon, build, workloads
-from parity import check_selection
+from parity import ATOL, RTOL, check_selection
 
 pytestmark = pytest.mark.gpu
 
@@ -73,7 +73,7 @@ def test_sweep_matches_oracle(name, over, budget):
             where = (j, var, r, l, h)
             swaps += check_selection(idx[j, r, l, h], o["idx"], o["S"], N, W, budget)
             g, want = float(lam[j, r, l, h]), o["lambda"]
-            assert abs(g - want) <= 1e-2 * abs(want) + 1e-6, (where, g, want)
+            assert abs(g - want) <= RTOL * abs(want) + ATOL, (where, g, want)
         assert swaps <= max_swaps, (var, swaps)
 
 
@@ -121,7 +121,7 @@ def test_sweep_sampled_oracle_at_gui_size():
     for j, res in enumerate(orc):
         for (r, l, h), o in res.items():
             check_selection(idx[j, r, l, h], o["idx"], o["S"], wl.seq_len, wl.window, budget)
-            assert abs(lam[j, r, l, h] - o["lambda"]) <= 1e-2 * abs(o["lambda"]) + 1e-6
+            assert abs(lam[j, r, l, h] - o["lambda"]) <= RTOL * abs(o["lambda"]) + ATOL
 
 
 def test_sweep_rejects_bad_variants():
