@@ -239,7 +239,9 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
     extern __shared__ __align__(16) float sm[];
     const Slots<T, PER> A1{sm};            // B (pooling), then E (coherence), then V
     const Slots<T, PER> A2{sm + T * PER};  // pooled backbone B~, then the final score S
-    __shared__ __align__(16) int hist[kSelHist];
+    // the selections never look at more than T PER keys
+    constexpr int kCap = T * PER < kSelCap ? T * PER : kSelCap;
+    __shared__ __align__(16) int hist[sel_hist_ints(kCap)];
     __shared__ int bcast[8];
     __shared__ int warp_sums[32];
     __shared__ float red[4 * 33];
@@ -392,7 +394,7 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
         if (M > 0) {
             // (the candidates' V sum rides on the selection's first reduction)
             float vtot = 0.f;
-            const SelectResult sel = radix_select_range(T * PER, M, SlotKeys<T, PER>{A2.a, n_cand},
+            const SelectResult sel = radix_select_range<kCap>(T * PER, M, SlotKeys<T, PER>{A2.a, n_cand},
                                                         hist, bcast, kmin, kmax, vsum, &vtot);
             const int eqb = ties_before(A2, i0, n_cand, sel, warp_sums, &total_s);
             const uint32_t mem = members(A2, i0, n_cand, sel, eqb);
@@ -454,7 +456,7 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
     if (keep >= n_cand) {
         for (int i = threadIdx.x; i < n_cand; i += blockDim.x) out[i] = i;
     } else if (keep > 0) {
-        const SelectResult sel = radix_select_range(T * PER, keep, SlotKeys<T, PER>{A2.a, n_cand},
+        const SelectResult sel = radix_select_range<kCap>(T * PER, keep, SlotKeys<T, PER>{A2.a, n_cand},
                                                     hist, bcast, skmin, skmax);
         const int eqb = ties_before(A2, i0, n_cand, sel, warp_sums, &total_s);
         const uint32_t mem = members(A2, i0, n_cand, sel, eqb);

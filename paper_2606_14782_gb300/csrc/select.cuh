@@ -29,13 +29,16 @@ struct SelectResult {
 };
 
 // Histogram bins of one select pass; the caller's shared array `hist` (16-
-// byte aligned) holds kSelHist ints: two bin buffers (passes alternate, so a
-// pass zeroes the next one's bins while it counts), 128 ints for the
-// reductions and the buffer counter, and a buffer of up to kSelCap keys.
+// byte aligned) holds sel_hist_ints(CAP) ints: two bin buffers (passes
+// alternate, so a pass zeroes the next one's bins while it counts), 128 ints
+// for the reductions and the buffer counter, and a buffer of up to CAP keys
+// (kSelCap, or fewer when a caller never selects among more keys: a smaller
+// array lets more CTAs share an SM).
 constexpr int kSelBits = 11;
 constexpr int kSelBins = 1 << kSelBits;
 constexpr int kSelCap = 2048;
-constexpr int kSelHist = 2 * kSelBins + 128 + kSelCap;
+__host__ __device__ constexpr int sel_hist_ints(int cap) { return 2 * kSelBins + 128 + cap; }
+constexpr int kSelHist = sel_hist_ints(kSelCap);
 
 // k-th best key over the included elements of [0, n) (1 <= k <= their
 // count).  First the range [kmin, kmax] of the included keys, then passes
@@ -50,7 +53,7 @@ constexpr int kSelHist = 2 * kSelBins + 128 + kSelCap;
 // key range (the callers know it from an earlier pass over the keys).  With
 // fsum, the block-wide sum of every thread's fval is reduced on the same
 // barriers and written to *fsum for every thread.
-template <typename KeyFn>
+template <int CAP = kSelCap, typename KeyFn>
 __device__ __noinline__ SelectResult radix_select_range(int n, int k, KeyFn key_of, int* hist, int* bcast,
                                            uint32_t kmin, uint32_t kmax, float fval = 0.f,
                                            float* fsum = nullptr)
@@ -98,13 +101,13 @@ __device__ __noinline__ SelectResult radix_select_range(int n, int k, KeyFn key_
     while (((span - 1u) >> shift) >= (uint64_t)kSelBins) ++shift;  // top bin index < kSelBins
     uint64_t width = span;  // keys of the current range: [lo, lo + width)
     int remaining = k;
-    // Once the current range holds at most kSelCap keys, the next pass also
+    // Once the current range holds at most CAP keys, the next pass also
     // copies them into the buffer and the passes after it read only that.
     int in_range = -1, nbuf = -1;  // unknown / not compacted
     for (int pass = 0;; ++pass) {
         int* const h = hist + (pass & 1) * kSelBins;          // zeroed
         int* const hn = hist + ((pass + 1) & 1) * kSelBins;   // the next pass's
-        const bool collect = nbuf < 0 && in_range >= 0 && in_range <= kSelCap;
+        const bool collect = nbuf < 0 && in_range >= 0 && in_range <= CAP;
         // the bins of the pass before this one were last read before the
         // barrier that ended it: free to zero for the next pass
         for (int b = threadIdx.x; b < kSelBins; b += blockDim.x) hn[b] = 0;
