@@ -360,7 +360,7 @@ template <int NV>
 __device__ __forceinline__ float max_tree(const float* v)
 {
     static_assert(NV == 32 || NV == 16, "32 or 16 logits");
-    if (NV == 32) {
+    if constexpr (NV == 32) {
         float m9[11];
 #pragma unroll
         for (int i = 0; i < 10; ++i) m9[i] = tc::max3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
@@ -370,11 +370,12 @@ __device__ __forceinline__ float max_tree(const float* v)
         const float mC = tc::max3(m9[6], m9[7], m9[8]);
         const float mD = fmaxf(m9[9], m9[10]);
         return fmaxf(tc::max3(mA, mB, mC), mD);
-    }
-    float m5[5];
+    } else {
+        float m5[5];
 #pragma unroll
-    for (int i = 0; i < 5; ++i) m5[i] = tc::max3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
-    return fmaxf(tc::max3(m5[0], m5[1], m5[2]), tc::max3(m5[3], m5[4], v[15]));
+        for (int i = 0; i < 5; ++i) m5[i] = tc::max3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+        return fmaxf(tc::max3(m5[0], m5[1], m5[2]), tc::max3(m5[3], m5[4], v[15]));
+    }
 }
 
 // Folds NV more logits of one row, whose maximum is mx, into its running

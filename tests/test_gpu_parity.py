@@ -337,7 +337,7 @@ def test_profile_hooks_count_launches(over, one_pass):
 
 # ------------------------------------------------ per-layer budgets (PyramidKV)
 
-def _compare_layer_budgets(wl, x, budgets, ko, vo, ix, orc):
+def _compare_layer_budgets(wl, x, budgets, ko, vo, ix, orc, log=None):
     N, W = wl.seq_len, wl.window
     kb = workloads.bf16_bits(x.k)
     vb = workloads.bf16_bits(x.v)
@@ -347,7 +347,7 @@ def _compare_layer_budgets(wl, x, budgets, ko, vo, ix, orc):
             continue
         r, l, h = key
         gi = ix[r][l][h].cpu().numpy()
-        swaps += check_selection(gi, o["idx"], o["S"], N, W, int(budgets[l]))
+        swaps += check_selection(gi, o["idx"], o["S"], N, W, int(budgets[l]), log=log, unit=key)
         Kc = ko[r][l][h].cpu().view(torch.int16).numpy().view(np.uint16)
         Vc = vo[r][l][h].cpu().view(torch.int16).numpy().view(np.uint16)
         assert np.array_equal(Kc, kb[r, l, h][gi]) and np.array_equal(Vc, vb[r, l, h][gi])
@@ -379,6 +379,44 @@ def test_pyramid_layer_budgets_parity(name, budget, beta):
     assert ix[0][0].shape[1] >= ix[0][-1].shape[1]
 
 
+PYRAMID_FULL = [("qwen-img", 512, 20), ("video", 652, 20), ("gui", 1024, 20)]
+
+
+@pytest.mark.parametrize("name,budget,beta", PYRAMID_FULL)
+def test_pyramid_layer_budgets_full_size(name, budget, beta):
+    """Per-layer budgets on the full-size launch (every request, layer and
+    kv-head in one call), every unit against the oracle: S element by
+    element, selections up to logged boundary swaps, gathers bit for bit."""
+    wl = workloads.CONFIGS[name]
+    x = workloads.generate(wl, seed=3, device="cuda")
+    budgets = bacon.pyramid_budgets(wl.layers, wl.window, budget, beta)
+    assert budgets == oracle.pyramid_budgets(wl.layers, wl.window, budget, beta).tolist()
+    p = bacon.default_params(keep_scores=1, max_seq_len=wl.seq_len, max_requests=wl.requests)
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool,
+                        budget, params=p)
+    ko, vo, ix = ctx.compress_layer_budgets(x.qwin, x.k, x.v, budgets)
+    ctx.sync()
+    R, Ly, H, N = wl.requests, wl.layers, wl.kv_heads, wl.seq_len
+    S = ctx.scores("S").cpu().numpy().reshape(R, Ly, H, N)
+    Bp = ctx.scores("Bpool").cpu().numpy().reshape(R, Ly, H, N)
+    ctx.close()
+    orc = oracle_run(wl, x, budgets)
+    units = [k for k in orc if isinstance(k, tuple)]
+    assert len(units) == R * Ly * H
+    for key in units:
+        check_scores(f"S {key}", S[key], orc[key]["S"])
+        check_scores(f"Bpool {key}", Bp[key], orc[key]["Bt"])
+    log = []
+    swaps = _compare_layer_budgets(wl, x, budgets, ko, vo, ix, orc, log=log)
+    record_swaps(f"{name} pyramid B={budget} beta={beta}", wl.name, [int(b) for b in budgets],
+                 len(units), [int(min(b, N)) - wl.window for b in budgets], log, "layer budgets")
+    assert swaps <= max(2, len(units) * (budget - wl.window) // 1000)
+    # budgets fall from the first layer to the last and are kept exactly
+    for r in range(R):
+        for l in range(Ly):
+            assert tuple(ix[r][l].shape) == (H, min(budgets[l], N))
+
+
 def test_uniform_layer_budgets_match_whole_step():
     wl = workloads.CONFIGS["tiny"].with_(layers=4, requests=2, seq_len=700, visual=(16, 650))
     x = workloads.generate(wl, seed=6, device="cuda")
@@ -402,12 +440,13 @@ def _head_threshold(S_cand, k):
     return S_cand[order[k - 1]] if k > 0 else np.inf
 
 
-@pytest.mark.parametrize("name,budget,alpha", [("tiny", 64, 0.2), ("tiny", 64, 1.0),
-                                               ("llava", 128, 0.2), ("qwen-img", 256, 0.0)])
-def test_adaptive_head_budgets_parity(name, budget, alpha):
-    base = workloads.CONFIGS[name]
-    wl = base.with_(layers=min(3, base.layers))
-    x = workloads.generate(wl, seed=8, device="cuda")
+def _adaptive_parity(wl, x, budget, alpha, case=None):
+    """AdaKV-style head budgets through the C ABI against the oracle at every
+    unit of the launch: S per token, per-head counts, each head's kept set
+    ascending with its window, K/V bit for bit, and the joint kept set of
+    each (request, layer) equal up to swaps whose oracle scores lie within
+    the tolerance of one of the thresholds that decide it (a head's
+    guaranteed-share boundary or the joint boundary).  Returns the swaps."""
     N, W, H = wl.seq_len, wl.window, wl.kv_heads
     p = bacon.default_params(keep_scores=1, max_seq_len=N, max_requests=wl.requests)
     ctx = bacon.Context(wl.layers, H, wl.q_heads, wl.head_dim, wl.window, wl.pool, budget,
@@ -418,11 +457,13 @@ def test_adaptive_head_budgets_parity(name, budget, alpha):
     ctx.close()
     ko, vo, ix, counts = ko.cpu(), vo.cpu(), ix.cpu().numpy(), counts.cpu().numpy()
     orc = oracle_run(wl, x, budget, adaptive_alpha=alpha)
+    assert len([k for k in orc if isinstance(k, tuple)]) == wl.requests * wl.layers * H
     kb = workloads.bf16_bits(x.k)
     vb = workloads.bf16_bits(x.v)
     K = min(budget, N) - W
     g = int(np.floor(alpha * K))
     swaps = 0
+    log = []
     for r in range(wl.requests):
         for l in range(wl.layers):
             cnt = counts[r, l]
@@ -445,11 +486,51 @@ def test_adaptive_head_budgets_parity(name, budget, alpha):
                 thresholds.append(_head_threshold(o["S"][:N - W], g))
             # joint threshold: the lowest oracle score among the oracle's picks
             thresholds.append(min(S_orc[t] for t in orc_sets))
-            for t in gpu_sets ^ orc_sets:
+            diff = sorted(gpu_sets ^ orc_sets)
+            worst = 0.0
+            for t in diff:
                 sv = S_orc[t]
-                assert min(abs(sv - th) for th in thresholds) <= 1e-5 + 2e-3 * abs(sv), (r, l, t, sv)
-            swaps += len(gpu_sets - orc_sets)
-    assert swaps <= max(2, wl.requests * wl.layers * H * K // 500)
+                gap = min(abs(sv - th) for th in thresholds)
+                assert gap <= 1e-5 + 2e-3 * abs(sv), (r, l, t, sv)
+                worst = max(worst, gap / (1e-5 + 2e-3 * abs(sv)))
+            extra = sorted(gpu_sets - orc_sets)
+            swaps += len(extra)
+            if diff:
+                missing = sorted(orc_sets - gpu_sets)
+                log.append({"unit": [r, l], "gpu_only": [list(t) for t in extra],
+                            "oracle_only": [list(t) for t in missing],
+                            "oracle_S_gpu_only": [float(S_orc[t]) for t in extra],
+                            "oracle_S_oracle_only": [float(S_orc[t]) for t in missing],
+                            "thresholds": [float(th) for th in thresholds],
+                            "max_gap_over_band": worst})
+    if case is not None:
+        record_swaps(case, wl.name, budget, wl.requests * wl.layers * H,
+                     f"{H * K} per (request, layer), shared by its heads", log,
+                     f"adaptive head budgets, alpha {alpha}")
+    return swaps
+
+
+@pytest.mark.parametrize("name,budget,alpha", [("tiny", 64, 0.2), ("tiny", 64, 1.0),
+                                               ("llava", 128, 0.2), ("qwen-img", 256, 0.0)])
+def test_adaptive_head_budgets_parity(name, budget, alpha):
+    base = workloads.CONFIGS[name]
+    wl = base.with_(layers=min(3, base.layers))
+    x = workloads.generate(wl, seed=8, device="cuda")
+    swaps = _adaptive_parity(wl, x, budget, alpha)
+    K = min(budget, wl.seq_len) - wl.window
+    assert swaps <= max(2, wl.requests * wl.layers * wl.kv_heads * K // 500)
+
+
+@pytest.mark.parametrize("name,budget,alpha", [("qwen-img", 512, 0.2), ("video", 652, 0.5),
+                                               ("gui", 1024, 0.2)])
+def test_adaptive_head_budgets_full_size(name, budget, alpha):
+    """The full-size launch (every request, layer and kv-head in one call),
+    every unit against the oracle, swaps logged."""
+    wl = workloads.CONFIGS[name]
+    x = workloads.generate(wl, seed=8, device="cuda")
+    swaps = _adaptive_parity(wl, x, budget, alpha, case=f"{name} adaptive B={budget} alpha={alpha}")
+    K = min(budget, wl.seq_len) - wl.window
+    assert swaps <= max(2, wl.requests * wl.layers * wl.kv_heads * K // 500)
 
 
 def test_adaptive_alpha_one_equals_uniform():
