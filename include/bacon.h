@@ -330,13 +330,12 @@ bacon_status bacon_profile_read(bacon_ctx* ctx, double* ms, int* launches, int n
  * after synchronising.
  *
  * The first call on a device looks up the array's device address (with
- * that device current) and caches it; make that first call before any
- * stream capture.  Every call uses the same array: calls whose work can
- * overlap on the GPU (different streams, or several host threads) race and
- * must be serialised by the caller.  The array keeps the last call's
- * contents; its error word, the one entry that must start at zero, is
- * cleared by each call on its stream, and every other entry a call reads
- * it has written first. */
+ * that device current) and caches it.  Every call uses the same array:
+ * calls whose work can overlap on the GPU (different streams, or several
+ * host threads) race and must be serialised by the caller.  The array keeps
+ * the last call's contents; its error word, the one entry that must start
+ * at zero, is cleared by each call on its stream, and every other entry a
+ * call reads it has written first. */
 bacon_status bacon_window_scores_noalloc(int kv_heads, int q_heads, int head_dim, int window,
                                          const void* q_win, const void* k, int seq_len,
                                          float* B_out, float* Q_out, float* E_out,
