@@ -50,6 +50,9 @@ def parse():
     ap.add_argument("--record-traffic", metavar="NCU_CSV", default=None,
                     help="store the DRAM bytes of an ncu --csv capture of this --config and "
                          "--requests in profiles/traffic.json, then exit")
+    ap.add_argument("--ncu-command", default=None,
+                    help="with --record-traffic: the ncu command line that wrote the log "
+                         "(stored beside the record)")
     return ap.parse_args()
 
 
@@ -435,7 +438,7 @@ def main():
         wl = workloads.CONFIGS[args.config]
         req = args.requests or wl.requests
         found = record_traffic(args.record_traffic, args.config, req,
-                               f"ncu log {os.path.basename(args.record_traffic)}")
+                               args.ncu_command or f"ncu log {os.path.basename(args.record_traffic)}")
         print(json.dumps({k: len(v[1]) for k, v in found.items()}))
         return
     if args.impl == "reference":
