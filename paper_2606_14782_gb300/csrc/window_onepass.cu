@@ -17,8 +17,10 @@
 //     butterfly transpose across the warp's lanes, meet at a CTA-wide
 //     mbarrier, write p = 2^(x - max) over the logits in TMEM while reducing
 //     the rows' sums of p the same way, meet again, and then each thread
-//     scales its token's p by 1 / (row sum x G W) and sums them over the rows
-//     (B) and over the last-position rows (Q), and stores E = [Q - B]_+.
+//     sums its token's p times 1 / (row sum x G W) over the rows (B) and
+//     over the last-position rows (Q), and stores E = [Q - B]_+.  Padding
+//     rows and the two row sets enter through per-row constants (a -inf
+//     shift, zero weights), so no row test runs per logit.
 // Every wait is bounded (abort flag, clock limit): on timeout the CTA records
 // BACON_ETIMEOUT, drains its own copies and MMAs, frees TMEM and returns.
 #include <cuda_bf16.h>
@@ -41,7 +43,7 @@ constexpr float kLog2e = 1.4426950408889634f;
 
 struct Layout {
     uint32_t q_half, q_slot, k_stage;  // bytes
-    uint32_t q, k, xr, xs, fm, bars, total;
+    uint32_t q, k, xr, xs, fm, fw, bars, total;
 };
 
 template <int D>
@@ -56,8 +58,9 @@ __host__ __device__ inline Layout layout()
     L.k = L.q + 2 * L.q_slot;
     L.xr = L.k + kStages * L.k_stage;             // [warp][row] partial maxima
     L.xs = L.xr + kEpiWarps * kRows * 4u;          // [warp][row] partial sums
-    L.fm = L.xs + kEpiWarps * kRows * 4u;          // [warp][row] the rows' max, then lse2
-    L.bars = L.fm + kEpiWarps * kRows * 4u;
+    L.fm = L.xs + kEpiWarps * kRows * 4u;          // [warp][row] -c max (this warp's copy)
+    L.fw = L.fm + kEpiWarps * kRows * 4u;          // [warp][row] (B weight, Q weight)
+    L.bars = L.fw + kEpiWarps * kRows * 8u;
     L.total = L.bars + 96u + 16u * kStages;
     return L;
 }
@@ -207,25 +210,22 @@ __device__ __forceinline__ float transpose_reduce(float* v)
     return v[0];
 }
 
-// Logits of one tile for this thread's token (its TMEM lane), scaled by c;
-// rows the token is hidden from are -inf: padding rows (bit r of `real` is
-// clear), tokens past N, and, in tiles that reach into the window, the rows
-// whose position precedes the token (row r sits at N - W + r mod W).
-__device__ __forceinline__ void load_row_logits(uint32_t taddr, const Shape& s, int tile, int tok,
-                                                float c, uint32_t real, float* v)
+// Raw logits of one tile for this thread's token (its TMEM lane); in tiles
+// that reach into the window (or past N) the rows the token is hidden from
+// become -inf: row r sits at position N - W + r mod W, and tokens past N are
+// hidden from every row.  Padding rows (beyond the unit's window rows) are
+// left as they are: their per-row constants below make every p of theirs 0.
+__device__ __forceinline__ void load_visible(uint32_t taddr, const Shape& s, int tile, int tok,
+                                             float* v)
 {
     tc::tmem_ld32(taddr, v);
     tc::tmem_ld_wait_regs32(v);
-    if (tile * kTok + kTok - 1 <= s.N - s.W) {  // whole tile before the window: no mask
-#pragma unroll
-        for (int r = 0; r < kRows; ++r) v[r] = (real >> r) & 1u ? v[r] * c : -INFINITY;
-        return;
-    }
+    if (tile * kTok + kTok - 1 <= s.N - s.W) return;  // whole tile before the window
     const int lim = tok < s.N ? tok - (s.N - s.W) : s.W;  // rows with r mod W < lim are hidden
     int rm = 0;                                            // r mod W
 #pragma unroll
     for (int r = 0; r < kRows; ++r) {
-        v[r] = ((real >> r) & 1u) && rm >= lim ? v[r] * c : -INFINITY;
+        if (rm < lim) v[r] = -INFINITY;
         rm = rm + 1 == s.W ? 0 : rm + 1;
     }
 }
@@ -245,14 +245,17 @@ __device__ void epilogue(const TcArgs& a, const Layout& L, uint8_t* sm, const Ba
     const Shape& s = a.s;
     const int ntiles = (s.N + kTok - 1) / kTok;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int ew = warp - 2;               // epilogue warp 0..15
+    const int ew = warp - 2;               // epilogue warp 0 .. kEpiWarps - 1
     const int quarter = warp & 3;          // TMEM lanes this warp may access
     const int group = ew >> 2;             // tiles t = group mod kGroups
     const uint32_t tl = tc::ld_shared(b.tmem_slot()) + ((uint32_t)(quarter * 32) << 16);
     float* xr = reinterpret_cast<float*>(sm + L.xr);
     float* xs = reinterpret_cast<float*>(sm + L.xs);
-    float* fm = reinterpret_cast<float*>(sm + L.fm) + ew * kRows;  // this warp's copy
+    // this warp's copies of the per-row constants
+    float* ncm = reinterpret_cast<float*>(sm + L.fm) + ew * kRows;     // -c max_r
+    float2* wbq = reinterpret_cast<float2*>(sm + L.fw) + ew * kRows;   // (B, Q) weights
     const float c = kLog2e * rsqrtf((float)D);
+    const unsigned long long c2 = tc::pack2(c, c);
     // bit r: row r is a window row / a last-position row (r mod W = W - 1)
     uint32_t real = 0u, last = 0u;
     for (int r = 0; r < kRows && r < s.rows; ++r) {
@@ -268,12 +271,13 @@ __device__ void epilogue(const TcArgs& a, const Layout& L, uint8_t* sm, const Ba
         if (!tc::mbar_wait(b.t_full(slot), use & 1, b.abort())) { ok = false; break; }
         tc::fence_after_sync();
         const uint32_t tbase = tl + slot * kSlotCols;
-        // (1) each row's maximum over the unit's tokens
+        // (1) each row's maximum logit over the unit's visible tokens (c > 0,
+        // so c max_r is the maximum of the scaled logits)
         float v[kRows], acc[kRows];
 #pragma unroll
         for (int r = 0; r < kRows; ++r) acc[r] = -INFINITY;
         for (int t = group; t < ntiles; t += kGroups) {
-            load_row_logits(tbase + t * kRows, s, t, t * kTok + quarter * 32 + lane, c, real, v);
+            load_visible(tbase + t * kRows, s, t, t * kTok + quarter * 32 + lane, v);
 #pragma unroll
             for (int r = 0; r < kRows; ++r) acc[r] = fmaxf(acc[r], v[r]);
         }
@@ -281,42 +285,58 @@ __device__ void epilogue(const TcArgs& a, const Layout& L, uint8_t* sm, const Ba
         if (!epi_sync(b, nsync)) { ok = false; break; }
         float mrow = -INFINITY;
         for (int w = 0; w < kEpiWarps; ++w) mrow = fmaxf(mrow, xr[w * kRows + lane]);
-        fm[lane] = mrow == -INFINITY ? 0.f : mrow;
+        // p = 2^(c x - c max_r); a padding row takes -inf, so all its p are 0
+        // (every window row sees at least the tokens before the window)
+        ncm[lane] = (real >> lane) & 1u ? -(c * mrow) : -INFINITY;
         __syncwarp();
-        // (2) each row's sum of p = 2^(x - max); p replaces the logit in TMEM
-        // (hidden tokens and padding rows give p = 0)
+        // (2) each row's sum of p; p replaces the logit in TMEM (hidden tokens
+        // give -inf, so p = 0)
+        unsigned long long acc2[kRows / 2];
 #pragma unroll
-        for (int r = 0; r < kRows; ++r) acc[r] = 0.f;
+        for (int r = 0; r < kRows / 2; ++r) acc2[r] = 0ull;
         for (int t = group; t < ntiles; t += kGroups) {
-            load_row_logits(tbase + t * kRows, s, t, t * kTok + quarter * 32 + lane, c, real, v);
+            load_visible(tbase + t * kRows, s, t, t * kTok + quarter * 32 + lane, v);
 #pragma unroll
-            for (int r = 0; r < kRows; ++r) {
-                v[r] = v[r] == -INFINITY ? 0.f : fast_exp2(v[r] - fm[r]);
-                acc[r] += v[r];
+            for (int r = 0; r < kRows; r += 2) {
+                const float2 nb = *reinterpret_cast<const float2*>(ncm + r);
+                const float2 x = tc::unpack2(tc::fma2(tc::pack2(v[r], v[r + 1]), c2,
+                                                      tc::pack2(nb.x, nb.y)));
+                v[r] = fast_exp2(x.x);
+                v[r + 1] = fast_exp2(x.y);
+                acc2[r >> 1] = tc::add2(acc2[r >> 1], tc::pack2(v[r], v[r + 1]));
             }
             tc::tmem_st32(tbase + t * kRows, v);
         }
         tc::tmem_st_wait();
+#pragma unroll
+        for (int r = 0; r < kRows; r += 2) {
+            const float2 z2 = tc::unpack2(acc2[r >> 1]);
+            acc[r] = z2.x;
+            acc[r + 1] = z2.y;
+        }
         xs[ew * kRows + lane] = transpose_reduce<false>(acc);
         if (!epi_sync(b, nsync)) { ok = false; break; }
         float z = 0.f;
         for (int w = 0; w < kEpiWarps; ++w) z += xs[w * kRows + lane];
-        // a token's share of row r is p / (Z_r G W) (= A / (G W)); padding rows 0
-        fm[lane] = z > 0.f ? 1.f / (z * (float)s.rows) : 0.f;
+        // a token's share of row r is p / (Z_r G W) (= A / (G W)): its weight
+        // in B, and in Q for the last-position rows; padding rows weigh 0
+        const float wr = z > 0.f ? 1.f / (z * (float)s.rows) : 0.f;
+        wbq[lane] = make_float2(wr, (last >> lane) & 1u ? wr : 0.f);
         __syncwarp();
-        // (3) the token's B (all rows), Q (last-position rows) and E
+        // (3) the token's B (all rows), Q (last-position rows) and E: one
+        // packed fma per row accumulates both
         for (int t = group; t < ntiles; t += kGroups) {
             const int tok = t * kTok + quarter * 32 + lane;
             tc::tmem_ld32(tbase + t * kRows, v);
             tc::tmem_ld_wait_regs32(v);
-            float bsum = 0.f, qsum = 0.f;
+            unsigned long long bq[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
             for (int r = 0; r < kRows; ++r) {
-                const float x = v[r] * fm[r];
-                bsum += x;
-                if ((last >> r) & 1u) qsum += x;
+                const float2 w2 = wbq[r];
+                bq[r & 3] = tc::fma2(tc::pack2(v[r], v[r]), tc::pack2(w2.x, w2.y), bq[r & 3]);
             }
-            qsum *= (float)s.W;
+            const float2 s2 = tc::unpack2(tc::add2(tc::add2(bq[0], bq[1]), tc::add2(bq[2], bq[3])));
+            const float bsum = s2.x, qsum = s2.y * (float)s.W;
             if (tok < s.N) {
                 const size_t idx = (size_t)u * s.N + tok;
                 a.B[idx] = bsum;
