@@ -307,7 +307,7 @@ def logged_swaps(path: str = SWAP_LOG_PATH):
     current = doc.get("code_sha256_16") == source_digest(names)
     cases = {k: {"swaps": v["swaps"], "units": v["units_checked"],
                  "selected_per_unit": v["selected_per_unit"],
-                 "max_gap_over_band": round(v["max_gap_over_band"], 3)}
+                 "max_gap_over_band": float(f"{v['max_gap_over_band']:.3g}")}
              for k, v in doc.get("cases", {}).items()
              if not k.startswith(("edge ", "fuzz "))}
     return {"source": "profiles/boundary_swaps.json", "current_code": current, "cases": cases}
