@@ -40,29 +40,9 @@ using namespace sel;
 // 16384 tokens and of 24 up to 24576.
 constexpr int kMaxPrompt = 24576;
 
-// Block-wide fp32 sum by a shuffle tree (pairwise, so the rounding error
-// grows with log2 of the count).  FP64 is avoided: its rate on this part is
-// a small fraction of fp32.
-__device__ float block_sum(float v, float* red)
-{
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    if (lane == 0) red[warp] = v;
-    __syncthreads();
-    if (warp == 0) {
-        float t = lane < (int)(blockDim.x >> 5) ? red[lane] : 0.f;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-        if (lane == 0) red[32] = t;
-    }
-    __syncthreads();
-    const float tot = red[32];
-    __syncthreads();
-    return tot;
-}
-
-// Four block-wide fp32 sums in one round (red holds 4 x 33 floats).
+// Four block-wide fp32 sums in one round (red holds 4 x 33 floats), by a
+// shuffle tree (pairwise, so the rounding error grows with log2 of the
+// count).  FP64 is avoided: its rate on this part is a small fraction of fp32.
 __device__ float4 block_sum4(float4 v, float* red)
 {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
