@@ -2,17 +2,20 @@
 
 It serves callers that cannot call cudaMalloc (for example a serving engine
 that has reserved all of HBM for its KV cache): its scratch is a static
-device array inside the library.  Its B, Q and E must agree with the context
-path (bacon_compress_all_layers + bacon_get_scores) within the parity
-tolerance, on two calls in a row that reuse the same static scratch.  This
-file is named so that pytest collects it last.
+device array inside the library.  Its B, Q and E must agree with the oracle
+(Eqs. 1, 2 and 4) and with the context path (bacon_compress_all_layers +
+bacon_get_scores) within the parity tolerance, on two calls in a row that
+reuse the same static scratch.  This file is named so that pytest collects
+it last.
 """
 
 import ctypes
 
+import numpy as np
 import pytest
 import torch
 
+import oracle
 from paper_2606_14782_gb300 import bacon, build, workloads
 from parity import check_scores
 
@@ -64,6 +67,27 @@ def test_noalloc_matches_context_path(lib, name, over):
         torch.cuda.synchronize()
         for kind in "BQE":
             check_scores(f"call {call} {kind}", out[kind].cpu().numpy(), ref[kind].numpy())
+
+
+@pytest.mark.parametrize("name,over", SHAPES, ids=[s[0] for s in SHAPES])
+def test_noalloc_matches_oracle(lib, name, over):
+    """Every kv-head of the layer against the oracle's Eqs. 1, 2 and 4."""
+    wl = workloads.CONFIGS["tiny"].with_(**over)
+    x = workloads.generate(wl, seed=7, device="cuda")
+    qwin, k = x.qwin[0, 0], x.k[0, 0]
+    out = {kind: torch.full((wl.kv_heads, wl.seq_len), float("nan"), device="cuda")
+           for kind in "BQE"}
+    assert _noalloc(lib, wl, qwin, k, out["B"], out["Q"], out["E"]) == bacon.BACON_OK
+    torch.cuda.synchronize()
+    qf = oracle.bf16_bits_to_f64(workloads.bf16_bits(qwin))
+    kf = oracle.bf16_bits_to_f64(workloads.bf16_bits(k))
+    G = wl.q_heads // wl.kv_heads
+    for h in range(wl.kv_heads):
+        B, Q = oracle.window_scores(qf[h * G:(h + 1) * G], kf[h])
+        E = oracle.residual(Q, B)
+        for kind, ref in (("B", B), ("Q", Q), ("E", E)):
+            check_scores(f"{name} kv-head {h} {kind}", out[kind][h].cpu().numpy(), ref)
+        assert np.isfinite(out["B"][h].cpu().numpy()).all()
 
 
 def test_noalloc_rejects_sizes_beyond_its_static_scratch(lib):
