@@ -508,7 +508,7 @@ def main():
     units = wl.requests * wl.layers * wl.kv_heads
     value = job_throughput(units, world, ms)
     hbm, tflops, tflops_sus, peak_src = peaks()
-    # a kernel timed inside a sub-second region runs at burst clocks: judge
+    # a kernel timed inside a sub-second region runs at burst clocks: compare
     # it against the burst bf16 peak; the sustained one is for a region of
     # seconds, where the power cap pulls the clocks down
     short = region_ms < 1000.0
