@@ -413,10 +413,14 @@ __device__ __forceinline__ void row_stats(const float* v, float mx, float c, uns
 // and a thread reads one of them and every other token of its 32 (16x64b
 // shape), so the two threads holding a row combine their statistics before
 // the merge.
-template <int D>
+template <int D, int J, bool H>
 __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, uint8_t* sm,
-                                               const Bars& b, int q_rows, int last_m64)
+                                               const Bars& b, int q_rows, int last_m64_rt)
 {
+    // J > 0: every tile has J jobs (J - 1 full blocks and the half block when
+    // H, else J full blocks), so a job's TMEM buffer and phase follow from the
+    // tile count at compile-time offsets; J = 0: counted at run time
+    const int last_m64 = J ? (H ? 1 : 0) : last_m64_rt;
     const Shape& s = a.s;
     const int ntiles = (s.N + kTileTok - 1) / kTileTok;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -425,7 +429,7 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
     const uint32_t tmem = tc::ld_shared(b.tmem_slot());
     float2* xchg = reinterpret_cast<float2*>(sm + L.xchg);  // [group][rb][128]
     const int nrb = (q_rows + 127) / 128;
-    const int nfull = last_m64 ? nrb - 1 : nrb;  // 128-row blocks
+    const int nfull = J ? (H ? J - 1 : J) : (last_m64 ? nrb - 1 : nrb);  // 128-row blocks
     // window row of this thread in the half block, and its tokens 2 c + odd
     const int row_h = nfull * 128 + quarter * 16 + (lane >> 2) + 8 * (lane & 1);
     const int odd = (lane >> 1) & 1;
@@ -433,8 +437,13 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
     const unsigned long long c2 = tc::pack2(c, c);
     int c0, c1;
     chunk_range(a.total_chunks, &c0, &c1);
-    int job = 0, nch = 0;
+    int job = 0, nch = 0, tcount = 0;
     bool ok = true;
+    // the last position each of this thread's rows sees (rows of every block)
+    int vis[4];
+#pragma unroll
+    for (int rb = 0; rb < 4; ++rb) vis[rb] = s.N - s.W + ((rb * 128 + quarter * 32 + lane) % s.W);
+    const int vis_h = s.N - s.W + (row_h % s.W);
     for (int g = c0; g < c1 && ok; ++g) {
         const int u = g / a.chunks, ci = g - u * a.chunks;
         // running statistics per 128-row block, and of the half block,
@@ -442,24 +451,23 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
         // logits only, whichever CTA and range of chunks processes it (every
         // launch shape gives the same bits)
         float m_run[4], z_run[4];
-        int vis[4];
 #pragma unroll
         for (int rb = 0; rb < 4; ++rb) {
             m_run[rb] = -INFINITY;
             z_run[rb] = 0.f;
-            vis[rb] = s.N - s.W + ((rb * 128 + quarter * 32 + lane) % s.W);
         }
         float m_h = -INFINITY, z_h = 0.f;
-        const int vis_h = s.N - s.W + (row_h % s.W);
         const int t1 = min(ntiles, (ci + 1) * kTilesPerChunk);
         for (int t = ci * kTilesPerChunk; t < t1 && ok; ++t) {
             const int tok0 = t * kTileTok + group * 32;
             const bool need_mask = tok0 + 31 > s.N - s.W;
+            const int jt0 = tcount * J;  // this tile's first job (J > 0)
+            ++tcount;
 #pragma unroll
             for (int rb = 0; rb < 4; ++rb) {
                 if (rb >= nfull) break;
-                const int buf = job & 3, nb = job >> 2;
-                ++job;
+                const int jj = J ? jt0 + rb : job++;
+                const int buf = jj & 3, nb = jj >> 2;
                 if (!tc::mbar_wait(b.t_full(buf), nb & 1, b.abort())) { ok = false; break; }
                 tc::fence_after_sync();
                 // the load also reduces the 32 logits to their maximum
@@ -480,8 +488,8 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
                 row_stats<32>(v, mx, c, c2, m_run[rb], z_run[rb]);
             }
             if (last_m64 && ok) {
-                const int buf = job & 3, nb = job >> 2;
-                ++job;
+                const int jj = J ? jt0 + (J - 1) : job++;
+                const int buf = jj & 3, nb = jj >> 2;
                 if (!tc::mbar_wait(b.t_full(buf), nb & 1, b.abort())) { ok = false; break; }
                 tc::fence_after_sync();
                 float v[16];
@@ -637,19 +645,22 @@ __device__ __forceinline__ void score_slice(float* v, int r0, int tok, const Sco
     }
 }
 
-template <bool FASTQ, bool MASK, int NBUF_LOG2>
-__device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int group, uint32_t tl,
-                                           const Bars& b, const ScoreCtx& k, int tok,
+// J > 0: every tile has J jobs and jt0 is this tile's first job, so a job's
+// TMEM buffer, phase and slice rotation follow at compile-time offsets;
+// J = 0: the jobs are counted at run time in `job`.
+template <bool FASTQ, bool MASK, int NBUF_LOG2, int J>
+__device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int jt0, int group,
+                                           uint32_t tl, const Bars& b, const ScoreCtx& k, int tok,
                                            unsigned long long* bacc, float& qacc)
 {
     const int lane = threadIdx.x & 31;
     constexpr uint32_t buf_cols = (uint32_t)kTmemCols >> NBUF_LOG2;
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-        if (j >= jt.n_jobs) break;
-        const int buf = job & ((1 << NBUF_LOG2) - 1), nb = job >> NBUF_LOG2;
-        const int sl = (group + job) & (kGroups - 1);
-        ++job;
+        if (j >= (J ? J : jt.n_jobs)) break;
+        const int jj = J ? jt0 + j : job++;
+        const int buf = jj & ((1 << NBUF_LOG2) - 1), nb = jj >> NBUF_LOG2;
+        const int sl = (group + jj) & (kGroups - 1);
         if (!tc::mbar_wait(b.t_full(buf), nb & 1, b.abort())) return false;
         tc::fence_after_sync();
         const int np = jt.n(j) >> 4, ns = (np + 1) >> 1;
@@ -704,7 +715,7 @@ __device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int gro
     return true;
 }
 
-template <int D, bool FASTQ, int NBUF_LOG2>
+template <int D, bool FASTQ, int NBUF_LOG2, int J>
 __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, uint8_t* sm,
                                                 const Bars& b, const JobTable& jt)
 {
@@ -736,8 +747,10 @@ __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, 
             unsigned long long bacc[2] = {0ull, 0ull};
             float qacc = 0.f;
             ok = need_mask
-                     ? score_tile<FASTQ, true, NBUF_LOG2>(jt, job, group, tl, b, k, tok, bacc, qacc)
-                     : score_tile<FASTQ, false, NBUF_LOG2>(jt, job, group, tl, b, k, tok, bacc, qacc);
+                     ? score_tile<FASTQ, true, NBUF_LOG2, J>(jt, job, ntile * J, group, tl, b, k, tok,
+                                                           bacc, qacc)
+                     : score_tile<FASTQ, false, NBUF_LOG2, J>(jt, job, ntile * J, group, tl, b, k, tok,
+                                                            bacc, qacc);
             if (!ok) break;
             const float2 b2 = tc::unpack2(tc::add2(bacc[0], bacc[1]));
             const float bsum = b2.x + b2.y;
@@ -897,13 +910,26 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, Plan p
         }
     } else {
         if (PASS == 1)
-            epilogue_stats<D>(a, L, sm, b, pl.q_rows, pl.last_m64);
-        else if (a.s.W % 16 == 0 && pl.nbuf_log2 == 1)
-            epilogue_scores<D, true, 1>(a, L, sm, b, jt);
-        else if (a.s.W % 16 == 0)
-            epilogue_scores<D, true, 2>(a, L, sm, b, jt);
+        {
+            const int nrb = (pl.q_rows + 127) / 128;
+            if (nrb == 4 && pl.last_m64)
+                epilogue_stats<D, 4, true>(a, L, sm, b, pl.q_rows, pl.last_m64);
+            else if (nrb == 2 && !pl.last_m64)
+                epilogue_stats<D, 2, false>(a, L, sm, b, pl.q_rows, pl.last_m64);
+            else
+                epilogue_stats<D, 0, false>(a, L, sm, b, pl.q_rows, pl.last_m64);
+        }
+        else if (a.s.W % 16 == 0 && pl.nbuf_log2 == 1) {
+            if (pl.n_jobs == 2)
+                epilogue_scores<D, true, 1, 2>(a, L, sm, b, jt);
+            else if (pl.n_jobs == 1)
+                epilogue_scores<D, true, 1, 1>(a, L, sm, b, jt);
+            else
+                epilogue_scores<D, true, 1, 0>(a, L, sm, b, jt);
+        } else if (a.s.W % 16 == 0)
+            epilogue_scores<D, true, 2, 0>(a, L, sm, b, jt);
         else  // W % 16 != 0: always four accumulators (see launch_impl)
-            epilogue_scores<D, false, 2>(a, L, sm, b, jt);
+            epilogue_scores<D, false, 2, 0>(a, L, sm, b, jt);
     }
 
     tc::fence_before_sync();
