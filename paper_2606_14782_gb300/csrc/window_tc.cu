@@ -383,27 +383,24 @@ __device__ __forceinline__ float max_tree(const float* v)
 // -inf.  (Exponentiating against the running maximum and redoing a job only
 // when its sum overflows would save the maximum but costs a data-dependent
 // branch per job, which measured slower than computing it.)
-template <int NV>
+template <int NV, bool MASKED = true>
 __device__ __forceinline__ void row_stats(const float* v, float mx, float c, unsigned long long c2,
                                           float& m_run, float& z_run)
 {
     const float m_new = fmaxf(m_run, mx * c);
-    if (m_new == -INFINITY) return;
+    if (MASKED && m_new == -INFINITY) return;
     const unsigned long long nm2 = tc::pack2(-m_new, -m_new);
-    unsigned long long acc[4] = {0ull, 0ull, 0ull, 0ull};
+    unsigned long long acc[2] = {0ull, 0ull};
 #pragma unroll
     for (int j = 0; j < NV; j += 2) {
         const float2 tt = tc::unpack2(tc::fma2(tc::pack2(v[j], v[j + 1]), c2, nm2));
-        acc[(j >> 1) & 3] = tc::add2(acc[(j >> 1) & 3], tc::pack2(fast_exp2(tt.x), fast_exp2(tt.y)));
+        acc[(j >> 1) & 1] = tc::add2(acc[(j >> 1) & 1], tc::pack2(fast_exp2(tt.x), fast_exp2(tt.y)));
     }
-    const float2 s2 = tc::unpack2(tc::add2(tc::add2(acc[0], acc[1]), tc::add2(acc[2], acc[3])));
+    const float2 s2 = tc::unpack2(tc::add2(acc[0], acc[1]));
     const float zs = s2.x + s2.y;
-    if (m_new > m_run) {
-        z_run = z_run * fast_exp2(m_run - m_new) + zs;
-        m_run = m_new;
-    } else {
-        z_run += zs;
-    }
+    // 2^0 = 1 when the maximum did not grow, 2^-inf = 0 for the first job
+    z_run = z_run * fast_exp2(m_run - m_new) + zs;
+    m_run = m_new;
 }
 
 // Thread = one window row (TMEM lane) x one 32-token quarter (its group) of
@@ -484,8 +481,10 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
                     for (int j = 0; j < 32; ++j)
                         if (tok0 + j > vis[rb]) v[j] = -INFINITY;
                     mx = max_tree<32>(v);
+                    row_stats<32, true>(v, mx, c, c2, m_run[rb], z_run[rb]);
+                } else {
+                    row_stats<32, false>(v, mx, c, c2, m_run[rb], z_run[rb]);
                 }
-                row_stats<32>(v, mx, c, c2, m_run[rb], z_run[rb]);
             }
             if (last_m64 && ok) {
                 const int jj = J ? jt0 + (J - 1) : job++;
@@ -647,8 +646,11 @@ __device__ __forceinline__ void score_slice(float* v, int r0, int tok, const Sco
 
 // J > 0: every tile has J jobs and jt0 is this tile's first job, so a job's
 // TMEM buffer, phase and slice rotation follow at compile-time offsets;
-// J = 0: the jobs are counted at run time in `job`.
-template <bool FASTQ, bool MASK, int NBUF_LOG2, int J>
+// J = 0: the jobs are counted at run time in `job`.  NPJ > 0: every job has
+// NPJ 16-row granules, so its slices' sizes and first rows are constants.
+// (Each instruction saved here is worth its share of the pass: the epilogue
+// is bound by instruction issue.)
+template <bool FASTQ, bool MASK, int NBUF_LOG2, int J, int NPJ>
 __device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int jt0, int group,
                                            uint32_t tl, const Bars& b, const ScoreCtx& k, int tok,
                                            unsigned long long* bacc, float& qacc)
@@ -663,7 +665,7 @@ __device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int jt0
         const int sl = (group + jj) & (kGroups - 1);
         if (!tc::mbar_wait(b.t_full(buf), nb & 1, b.abort())) return false;
         tc::fence_after_sync();
-        const int np = jt.n(j) >> 4, ns = (np + 1) >> 1;
+        const int np = NPJ ? NPJ : jt.n(j) >> 4, ns = (np + 1) >> 1;
         // this group's 32-column slices of the job: sl, sl + 4, ...; the
         // buffer is released once the last of them is in registers
         const int mine = sl < ns ? (sl + kGroups < ns ? 2 : 1) : 0;
@@ -672,11 +674,14 @@ __device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int jt0
             __syncwarp();
             if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
         }
-        for (int q = 0; q < mine; ++q) {
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            if (q >= mine) break;
             const int sx = sl + kGroups * q;
             const uint32_t taddr = tl + buf * buf_cols + 32 * sx;
-            const int r0 = jt.row0(j) + 32 * sx;
-            const bool two = 2 * sx + 1 < np, last = q + 1 == mine;
+            const int r0 = (NPJ ? 16 * NPJ * j : jt.row0(j)) + 32 * sx;
+            const bool two = (NPJ && NPJ % 2 == 0) ? true : 2 * sx + 1 < np;
+            const bool last = q + 1 == mine;
             if (!MASK) {
                 float v[32];
                 if (two) {
@@ -715,7 +720,7 @@ __device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int jt0
     return true;
 }
 
-template <int D, bool FASTQ, int NBUF_LOG2, int J>
+template <int D, bool FASTQ, int NBUF_LOG2, int J, int NPJ>
 __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, uint8_t* sm,
                                                 const Bars& b, const JobTable& jt)
 {
@@ -747,10 +752,10 @@ __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, 
             unsigned long long bacc[2] = {0ull, 0ull};
             float qacc = 0.f;
             ok = need_mask
-                     ? score_tile<FASTQ, true, NBUF_LOG2, J>(jt, job, ntile * J, group, tl, b, k, tok,
-                                                           bacc, qacc)
-                     : score_tile<FASTQ, false, NBUF_LOG2, J>(jt, job, ntile * J, group, tl, b, k, tok,
-                                                            bacc, qacc);
+                     ? score_tile<FASTQ, true, NBUF_LOG2, J, NPJ>(jt, job, ntile * J, group, tl, b, k,
+                                                                tok, bacc, qacc)
+                     : score_tile<FASTQ, false, NBUF_LOG2, J, NPJ>(jt, job, ntile * J, group, tl, b, k,
+                                                                 tok, bacc, qacc);
             if (!ok) break;
             const float2 b2 = tc::unpack2(tc::add2(bacc[0], bacc[1]));
             const float bsum = b2.x + b2.y;
@@ -920,16 +925,20 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, Plan p
                 epilogue_stats<D, 0, false>(a, L, sm, b, pl.q_rows, pl.last_m64);
         }
         else if (a.s.W % 16 == 0 && pl.nbuf_log2 == 1) {
-            if (pl.n_jobs == 2)
-                epilogue_scores<D, true, 1, 2>(a, L, sm, b, jt);
+            if (pl.n_jobs == 2 && pl.granules == 28)
+                epilogue_scores<D, true, 1, 2, 14>(a, L, sm, b, jt);
+            else if (pl.n_jobs == 2)
+                epilogue_scores<D, true, 1, 2, 0>(a, L, sm, b, jt);
+            else if (pl.n_jobs == 1 && pl.granules == 14)
+                epilogue_scores<D, true, 1, 1, 14>(a, L, sm, b, jt);
             else if (pl.n_jobs == 1)
-                epilogue_scores<D, true, 1, 1>(a, L, sm, b, jt);
+                epilogue_scores<D, true, 1, 1, 0>(a, L, sm, b, jt);
             else
-                epilogue_scores<D, true, 1, 0>(a, L, sm, b, jt);
+                epilogue_scores<D, true, 1, 0, 0>(a, L, sm, b, jt);
         } else if (a.s.W % 16 == 0)
-            epilogue_scores<D, true, 2, 0>(a, L, sm, b, jt);
+            epilogue_scores<D, true, 2, 0, 0>(a, L, sm, b, jt);
         else  // W % 16 != 0: always four accumulators (see launch_impl)
-            epilogue_scores<D, false, 2, 0>(a, L, sm, b, jt);
+            epilogue_scores<D, false, 2, 0, 0>(a, L, sm, b, jt);
     }
 
     tc::fence_before_sync();
