@@ -593,7 +593,9 @@ struct ScoreCtx {
     uint32_t qmask;  // bit g: 16-row granule g ends on a last-position row
 };
 
-template <int NC, bool FASTQ, bool MASK>
+// WQ > 0: the window W (a multiple of 16) as a constant, so a granule's
+// last-position test is a mask of its first row instead of a table lookup.
+template <int NC, bool FASTQ, bool MASK, int WQ = 0>
 __device__ __forceinline__ void score_slice(float* v, int r0, int tok, const ScoreCtx& k,
                                             unsigned long long* bacc, float& qacc)
 {
@@ -639,8 +641,10 @@ __device__ __forceinline__ void score_slice(float* v, int r0, int tok, const Sco
         // with W a multiple of 16 only a granule's last row can be a
         // last-position row: one mask test per granule, after the loop
 #pragma unroll
-        for (int g = 0; g < NC / 16; ++g)
-            if ((k.qmask >> ((r0 >> 4) + g)) & 1u) qacc += q_end[g];
+        for (int g = 0; g < NC / 16; ++g) {
+            const bool last_row = WQ ? (r0 + 16 * g + 16) % WQ == 0 : ((k.qmask >> ((r0 >> 4) + g)) & 1u);
+            if (last_row) qacc += q_end[g];
+        }
     }
 }
 
@@ -650,7 +654,7 @@ __device__ __forceinline__ void score_slice(float* v, int r0, int tok, const Sco
 // NPJ 16-row granules, so its slices' sizes and first rows are constants.
 // (Each instruction saved here is worth its share of the pass: the epilogue
 // is bound by instruction issue.)
-template <bool FASTQ, bool MASK, int NBUF_LOG2, int J, int NPJ>
+template <bool FASTQ, bool MASK, int NBUF_LOG2, int J, int NPJ, int WQ>
 __device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int jt0, int group,
                                            uint32_t tl, const Bars& b, const ScoreCtx& k, int tok,
                                            unsigned long long* bacc, float& qacc)
@@ -697,9 +701,9 @@ __device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int jt0
                     if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
                 }
                 if (two)
-                    score_slice<32, FASTQ, false>(v, r0, tok, k, bacc, qacc);
+                    score_slice<32, FASTQ, false, WQ>(v, r0, tok, k, bacc, qacc);
                 else
-                    score_slice<16, FASTQ, false>(v, r0, tok, k, bacc, qacc);
+                    score_slice<16, FASTQ, false, WQ>(v, r0, tok, k, bacc, qacc);
             } else {
                 // tiles that reach into the window (one or two per unit) go
                 // 16 columns at a time, keeping the masking's register demand low
@@ -707,7 +711,7 @@ __device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int jt0
                 for (int h = 0; h < (two ? 2 : 1); ++h) {
                     tc::tmem_ld16(taddr + 16 * h, v);
                     tc::tmem_ld_wait_regs16(v);
-                    score_slice<16, FASTQ, true>(v, r0 + 16 * h, tok, k, bacc, qacc);
+                    score_slice<16, FASTQ, true, WQ>(v, r0 + 16 * h, tok, k, bacc, qacc);
                 }
                 if (last) {
                     tc::fence_before_sync();
@@ -720,7 +724,7 @@ __device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int jt0
     return true;
 }
 
-template <int D, bool FASTQ, int NBUF_LOG2, int J, int NPJ>
+template <int D, bool FASTQ, int NBUF_LOG2, int J, int NPJ, int WQ = 0>
 __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, uint8_t* sm,
                                                 const Bars& b, const JobTable& jt)
 {
@@ -752,10 +756,10 @@ __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, 
             unsigned long long bacc[2] = {0ull, 0ull};
             float qacc = 0.f;
             ok = need_mask
-                     ? score_tile<FASTQ, true, NBUF_LOG2, J, NPJ>(jt, job, ntile * J, group, tl, b, k,
-                                                                tok, bacc, qacc)
-                     : score_tile<FASTQ, false, NBUF_LOG2, J, NPJ>(jt, job, ntile * J, group, tl, b, k,
-                                                                 tok, bacc, qacc);
+                     ? score_tile<FASTQ, true, NBUF_LOG2, J, NPJ, WQ>(jt, job, ntile * J, group, tl, b,
+                                                                    k, tok, bacc, qacc)
+                     : score_tile<FASTQ, false, NBUF_LOG2, J, NPJ, WQ>(jt, job, ntile * J, group, tl, b,
+                                                                     k, tok, bacc, qacc);
             if (!ok) break;
             const float2 b2 = tc::unpack2(tc::add2(bacc[0], bacc[1]));
             const float bsum = b2.x + b2.y;
@@ -925,10 +929,14 @@ __global__ void __launch_bounds__(kThreads, 1) window_tc_kernel(TcArgs a, Plan p
                 epilogue_stats<D, 0, false>(a, L, sm, b, pl.q_rows, pl.last_m64);
         }
         else if (a.s.W % 16 == 0 && pl.nbuf_log2 == 1) {
-            if (pl.n_jobs == 2 && pl.granules == 28)
+            if (pl.n_jobs == 2 && pl.granules == 28 && a.s.W == 64)
+                epilogue_scores<D, true, 1, 2, 14, 64>(a, L, sm, b, jt);
+            else if (pl.n_jobs == 2 && pl.granules == 28)
                 epilogue_scores<D, true, 1, 2, 14>(a, L, sm, b, jt);
             else if (pl.n_jobs == 2)
                 epilogue_scores<D, true, 1, 2, 0>(a, L, sm, b, jt);
+            else if (pl.n_jobs == 1 && pl.granules == 14 && a.s.W == 32)
+                epilogue_scores<D, true, 1, 1, 14, 32>(a, L, sm, b, jt);
             else if (pl.n_jobs == 1 && pl.granules == 14)
                 epilogue_scores<D, true, 1, 1, 14>(a, L, sm, b, jt);
             else if (pl.n_jobs == 1)
