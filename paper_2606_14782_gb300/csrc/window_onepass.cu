@@ -215,18 +215,18 @@ __device__ __forceinline__ float transpose_reduce(float* v)
 // become -inf: row r sits at position N - W + r mod W, and tokens past N are
 // hidden from every row.  Padding rows (beyond the unit's window rows) are
 // left as they are: their per-row constants below make every p of theirs 0.
-__device__ __forceinline__ void load_visible(uint32_t taddr, const Shape& s, int tile, int tok,
+__device__ __forceinline__ void load_visible(uint32_t taddr, int N, int W, int tile, int tok,
                                              float* v)
 {
     tc::tmem_ld32(taddr, v);
     tc::tmem_ld_wait_regs32(v);
-    if (tile * kTok + kTok - 1 <= s.N - s.W) return;  // whole tile before the window
-    const int lim = tok < s.N ? tok - (s.N - s.W) : s.W;  // rows with r mod W < lim are hidden
-    int rm = 0;                                            // r mod W
+    if (tile * kTok + kTok - 1 <= N - W) return;  // whole tile before the window
+    const int lim = tok < N ? tok - (N - W) : W;  // rows with r mod W < lim are hidden
+    int rm = 0;                                    // r mod W
 #pragma unroll
     for (int r = 0; r < kRows; ++r) {
         if (rm < lim) v[r] = -INFINITY;
-        rm = rm + 1 == s.W ? 0 : rm + 1;
+        rm = rm + 1 == W ? 0 : rm + 1;
     }
 }
 
@@ -239,11 +239,17 @@ __device__ __forceinline__ bool epi_sync(const Bars& b, int& nsync)
     return ok;
 }
 
-template <int D>
+// SPEC: the multi-head 1024-token unit (N = 1024, W = 32, 32 window rows)
+// with its sizes as constants: the tile loops unroll and the mask test runs
+// only where a tile can reach into the window (every instruction saved counts:
+// the epilogue is bound by instruction issue).
+template <int D, bool SPEC>
 __device__ void epilogue(const TcArgs& a, const Layout& L, uint8_t* sm, const Bars& b)
 {
     const Shape& s = a.s;
-    const int ntiles = (s.N + kTok - 1) / kTok;
+    const int N = SPEC ? 1024 : s.N, W = SPEC ? 32 : s.W, rows = SPEC ? kRows : s.rows;
+    const int ntiles = (N + kTok - 1) / kTok;
+    constexpr int kSpecPerGroup = 1024 / kTok / kGroups;  // tiles per group (SPEC)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int ew = warp - 2;               // epilogue warp 0 .. kEpiWarps - 1
     const int quarter = warp & 3;          // TMEM lanes this warp may access
@@ -258,9 +264,9 @@ __device__ void epilogue(const TcArgs& a, const Layout& L, uint8_t* sm, const Ba
     const unsigned long long c2 = tc::pack2(c, c);
     // bit r: row r is a window row / a last-position row (r mod W = W - 1)
     uint32_t real = 0u, last = 0u;
-    for (int r = 0; r < kRows && r < s.rows; ++r) {
+    for (int r = 0; r < kRows && r < rows; ++r) {
         real |= 1u << r;
-        if (r % s.W == s.W - 1) last |= 1u << r;
+        if (r % W == W - 1) last |= 1u << r;
     }
     int u0, u1;
     unit_range(s.units, &u0, &u1);
@@ -276,8 +282,11 @@ __device__ void epilogue(const TcArgs& a, const Layout& L, uint8_t* sm, const Ba
         float v[kRows], acc[kRows];
 #pragma unroll
         for (int r = 0; r < kRows; ++r) acc[r] = -INFINITY;
-        for (int t = group; t < ntiles; t += kGroups) {
-            load_visible(tbase + t * kRows, s, t, t * kTok + quarter * 32 + lane, v);
+#pragma unroll
+        for (int i = 0; i < (SPEC ? kSpecPerGroup : kMaxTiles / kGroups); ++i) {
+            const int t = group + kGroups * i;
+            if (!SPEC && t >= ntiles) break;
+            load_visible(tbase + t * kRows, N, W, t, t * kTok + quarter * 32 + lane, v);
 #pragma unroll
             for (int r = 0; r < kRows; ++r) acc[r] = fmaxf(acc[r], v[r]);
         }
@@ -294,8 +303,11 @@ __device__ void epilogue(const TcArgs& a, const Layout& L, uint8_t* sm, const Ba
         unsigned long long acc2[kRows / 2];
 #pragma unroll
         for (int r = 0; r < kRows / 2; ++r) acc2[r] = 0ull;
-        for (int t = group; t < ntiles; t += kGroups) {
-            load_visible(tbase + t * kRows, s, t, t * kTok + quarter * 32 + lane, v);
+#pragma unroll
+        for (int i = 0; i < (SPEC ? kSpecPerGroup : kMaxTiles / kGroups); ++i) {
+            const int t = group + kGroups * i;
+            if (!SPEC && t >= ntiles) break;
+            load_visible(tbase + t * kRows, N, W, t, t * kTok + quarter * 32 + lane, v);
 #pragma unroll
             for (int r = 0; r < kRows; r += 2) {
                 const float2 nb = *reinterpret_cast<const float2*>(ncm + r);
@@ -320,12 +332,15 @@ __device__ void epilogue(const TcArgs& a, const Layout& L, uint8_t* sm, const Ba
         for (int w = 0; w < kEpiWarps; ++w) z += xs[w * kRows + lane];
         // a token's share of row r is p / (Z_r G W) (= A / (G W)): its weight
         // in B, and in Q for the last-position rows; padding rows weigh 0
-        const float wr = z > 0.f ? 1.f / (z * (float)s.rows) : 0.f;
+        const float wr = z > 0.f ? 1.f / (z * (float)rows) : 0.f;
         wbq[lane] = make_float2(wr, (last >> lane) & 1u ? wr : 0.f);
         __syncwarp();
         // (3) the token's B (all rows), Q (last-position rows) and E: one
         // packed fma per row accumulates both
-        for (int t = group; t < ntiles; t += kGroups) {
+#pragma unroll
+        for (int i = 0; i < (SPEC ? kSpecPerGroup : kMaxTiles / kGroups); ++i) {
+            const int t = group + kGroups * i;
+            if (!SPEC && t >= ntiles) break;
             const int tok = t * kTok + quarter * 32 + lane;
             tc::tmem_ld32(tbase + t * kRows, v);
             tc::tmem_ld_wait_regs32(v);
@@ -336,9 +351,9 @@ __device__ void epilogue(const TcArgs& a, const Layout& L, uint8_t* sm, const Ba
                 bq[r & 3] = tc::fma2(tc::pack2(v[r], v[r]), tc::pack2(w2.x, w2.y), bq[r & 3]);
             }
             const float2 s2 = tc::unpack2(tc::add2(tc::add2(bq[0], bq[1]), tc::add2(bq[2], bq[3])));
-            const float bsum = s2.x, qsum = s2.y * (float)s.W;
-            if (tok < s.N) {
-                const size_t idx = (size_t)u * s.N + tok;
+            const float bsum = s2.x, qsum = s2.y * (float)W;
+            if (tok < N) {
+                const size_t idx = (size_t)u * N + tok;
                 a.B[idx] = bsum;
                 a.Q[idx] = qsum;
                 a.E[idx] = fmaxf(qsum - bsum, 0.f);
@@ -351,7 +366,7 @@ __device__ void epilogue(const TcArgs& a, const Layout& L, uint8_t* sm, const Ba
     if (!ok) raise_abort(b, a.err);
 }
 
-template <int D>
+template <int D, bool SPEC>
 __global__ void __launch_bounds__(kThreads, 1) window_onepass_kernel(TcArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
@@ -390,7 +405,7 @@ __global__ void __launch_bounds__(kThreads, 1) window_onepass_kernel(TcArgs a)
     else if (warp == 1) {
         if (tc::elect_one()) issue<D>(a, L, sm, b);
     } else {
-        epilogue<D>(a, L, sm, b);
+        epilogue<D, SPEC>(a, L, sm, b);
     }
 
     tc::fence_before_sync();
@@ -410,18 +425,18 @@ int num_sms_onepass()
     return n > 0 ? n : 1;
 }
 
-template <int D>
+template <int D, bool SPEC>
 cudaError_t launch_d(const TcArgs& a, cudaStream_t st)
 {
     const Layout L = layout<D>();
     size_t bytes = L.total + 1024;
     if (bytes < 116 * 1024) bytes = 116 * 1024;  // one CTA (one TMEM allocation) per SM
-    cudaError_t e = cudaFuncSetAttribute(window_onepass_kernel<D>,
+    cudaError_t e = cudaFuncSetAttribute(window_onepass_kernel<D, SPEC>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
     if (e != cudaSuccess) return e;
     const int sms = num_sms_onepass();
     const int grid = a.s.units < sms ? a.s.units : sms;
-    window_onepass_kernel<D><<<grid, kThreads, bytes, st>>>(a);
+    window_onepass_kernel<D, SPEC><<<grid, kThreads, bytes, st>>>(a);
     return cudaGetLastError();
 }
 
@@ -435,7 +450,9 @@ bool window_onepass_fits(const Shape& s)
 cudaError_t launch_window_onepass(const TcArgs& a, cudaStream_t st)
 {
     if (!window_onepass_fits(a.s)) return cudaErrorInvalidValue;
-    return a.s.d == 128 ? launch_d<128>(a, st) : launch_d<64>(a, st);
+    const bool spec = a.s.N == 1024 && a.s.W == 32 && a.s.rows == kRows;
+    if (a.s.d == 128) return spec ? launch_d<128, true>(a, st) : launch_d<128, false>(a, st);
+    return spec ? launch_d<64, true>(a, st) : launch_d<64, false>(a, st);
 }
 
 }  // namespace bacon
