@@ -678,45 +678,71 @@ __device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int jt0
             __syncwarp();
             if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
         }
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-            if (q >= mine) break;
-            const int sx = sl + kGroups * q;
-            const uint32_t taddr = tl + buf * buf_cols + 32 * sx;
-            const int r0 = (NPJ ? 16 * NPJ * j : jt.row0(j)) + 32 * sx;
-            const bool two = (NPJ && NPJ % 2 == 0) ? true : 2 * sx + 1 < np;
-            const bool last = q + 1 == mine;
-            if (!MASK) {
-                float v[32];
-                if (two) {
-                    tc::tmem_ld32(taddr, v);
-                    tc::tmem_ld_wait_regs32(v);
-                } else {
-                    tc::tmem_ld16(taddr, v);
-                    tc::tmem_ld_wait_regs16(v);
-                }
-                if (last) {
-                    tc::fence_before_sync();
-                    __syncwarp();
-                    if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
-                }
-                if (two)
-                    score_slice<32, FASTQ, false, WQ>(v, r0, tok, k, bacc, qacc);
-                else
-                    score_slice<16, FASTQ, false, WQ>(v, r0, tok, k, bacc, qacc);
+        if constexpr (NPJ == 14 && !MASK) {
+            // 224 columns: the group of rotation sl takes columns [64 sl,
+            // 64 sl + 64) (the last one [192, 224)) in one load pair and
+            // releases the buffer once (fewer instructions per column)
+            const uint32_t tb = tl + buf * buf_cols + 64 * sl;
+            const int r0 = 16 * NPJ * j + 64 * sl;
+            if (sl < 3) {
+                float v[64];
+                tc::tmem_ld32(tb, v);
+                tc::tmem_ld32(tb + 32, v + 32);
+                tc::tmem_ld_wait_regs32(v);
+                tc::tmem_ld_wait_regs32(v + 32);
+                tc::fence_before_sync();
+                __syncwarp();
+                if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
+                score_slice<32, FASTQ, false, WQ>(v, r0, tok, k, bacc, qacc);
+                score_slice<32, FASTQ, false, WQ>(v + 32, r0 + 32, tok, k, bacc, qacc);
             } else {
-                // tiles that reach into the window (one or two per unit) go
-                // 16 columns at a time, keeping the masking's register demand low
-                float v[16];
-                for (int h = 0; h < (two ? 2 : 1); ++h) {
-                    tc::tmem_ld16(taddr + 16 * h, v);
-                    tc::tmem_ld_wait_regs16(v);
-                    score_slice<16, FASTQ, true, WQ>(v, r0 + 16 * h, tok, k, bacc, qacc);
-                }
-                if (last) {
-                    tc::fence_before_sync();
-                    __syncwarp();
-                    if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
+                float v[32];
+                tc::tmem_ld32(tb, v);
+                tc::tmem_ld_wait_regs32(v);
+                tc::fence_before_sync();
+                __syncwarp();
+                if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
+                score_slice<32, FASTQ, false, WQ>(v, r0, tok, k, bacc, qacc);
+            }
+        } else {
+            for (int q = 0; q < mine; ++q) {
+                const int sx = sl + kGroups * q;
+                const uint32_t taddr = tl + buf * buf_cols + 32 * sx;
+                const int r0 = (NPJ ? 16 * NPJ * j : jt.row0(j)) + 32 * sx;
+                const bool two = (NPJ && NPJ % 2 == 0) ? true : 2 * sx + 1 < np;
+                const bool last = q + 1 == mine;
+                if (!MASK) {
+                    float v[32];
+                    if (two) {
+                        tc::tmem_ld32(taddr, v);
+                        tc::tmem_ld_wait_regs32(v);
+                    } else {
+                        tc::tmem_ld16(taddr, v);
+                        tc::tmem_ld_wait_regs16(v);
+                    }
+                    if (last) {
+                        tc::fence_before_sync();
+                        __syncwarp();
+                        if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
+                    }
+                    if (two)
+                        score_slice<32, FASTQ, false, WQ>(v, r0, tok, k, bacc, qacc);
+                    else
+                        score_slice<16, FASTQ, false, WQ>(v, r0, tok, k, bacc, qacc);
+                } else {
+                    // tiles that reach into the window (one or two per unit) go
+                    // 16 columns at a time, keeping the masking's register demand low
+                    float v[16];
+                    for (int h = 0; h < (two ? 2 : 1); ++h) {
+                        tc::tmem_ld16(taddr + 16 * h, v);
+                        tc::tmem_ld_wait_regs16(v);
+                        score_slice<16, FASTQ, true, WQ>(v, r0 + 16 * h, tok, k, bacc, qacc);
+                    }
+                    if (last) {
+                        tc::fence_before_sync();
+                        __syncwarp();
+                        if (lane == 0) tc::mbar_arrive(b.t_empty(buf));
+                    }
                 }
             }
         }
