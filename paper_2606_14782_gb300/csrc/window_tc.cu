@@ -18,11 +18,15 @@
 //                  256-column accumulators (four of 128 when shared memory
 //                  is short); the accumulator starts from each row's
 //                  -lse2 / c (one extra MMA against a constant operand) and
-//                  a thread owns one token and 32-column slices of a job.
+//                  a thread owns one token and a share of a job's columns
+//                  (32-column slices, or one 64-column range of a 224-column
+//                  job).
 // Each CTA takes a contiguous range of 1024-token chunks of the flattened
 // (unit, chunk) space, so it reloads the window rows only when its range
 // crosses into the next (request, layer, kv-head).  The epilogue groups meet
 // through shared-memory slots and arrival counters, never at a barrier.
+// The epilogues are bound by instruction issue, so the common plans are
+// compiled with their job counts, job sizes and window as constants.
 // Every wait is bounded: on timeout the CTA raises an abort flag, records
 // kErrTimeout in the error word, drains its own copies and MMAs, frees TMEM
 // and returns.
@@ -584,8 +588,9 @@ __device__ __forceinline__ void epilogue_stats(const TcArgs& a, const Smem& L, u
 // Thread = one token (TMEM lane).  The accumulator of a job already holds
 // logit - lse2 / c for each of its window rows (columns), so a column's share
 // of B is 2^(c D) (= A_{q,i} / (G W)).  Each job's columns are cut into
-// 32-column slices, one per group, rotated from job to job so that the short
-// last slice moves between the groups.  Q sums the columns of last-position
+// 32-column slices, one per group (a 224-column job into 64-column ranges),
+// rotated from job to job so that the short last share moves between the
+// groups.  Q sums the columns of last-position
 // rows (scaled by W at the end, so that the G heads' rows average to Q).
 struct ScoreCtx {
     unsigned long long c2;
