@@ -660,9 +660,9 @@ __device__ __forceinline__ void score_slice(float* v, int r0, int tok, const Sco
 // (Each instruction saved here is worth its share of the pass: the epilogue
 // is bound by instruction issue.)
 template <bool FASTQ, bool MASK, int NBUF_LOG2, int J, int NPJ, int WQ>
-__device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int jt0, int group,
-                                           uint32_t tl, const Bars& b, const ScoreCtx& k, int tok,
-                                           unsigned long long* bacc, float& qacc)
+__device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int jt0, int rot0,
+                                           int group, uint32_t tl, const Bars& b, const ScoreCtx& k,
+                                           int tok, unsigned long long* bacc, float& qacc)
 {
     const int lane = threadIdx.x & 31;
     constexpr uint32_t buf_cols = (uint32_t)kTmemCols >> NBUF_LOG2;
@@ -671,7 +671,10 @@ __device__ __forceinline__ bool score_tile(const JobTable& jt, int& job, int jt0
         if (j >= (J ? J : jt.n_jobs)) break;
         const int jj = J ? jt0 + j : job++;
         const int buf = jj & ((1 << NBUF_LOG2) - 1), nb = jj >> NBUF_LOG2;
-        const int sl = (group + jj) & (kGroups - 1);
+        // the share rotation follows the tile's own index (rot0), not the
+        // CTA's job count, so every launch shape sums a token's columns in
+        // the same order (the same bits)
+        const int sl = (group + rot0 + j) & (kGroups - 1);
         if (!tc::mbar_wait(b.t_full(buf), nb & 1, b.abort())) return false;
         tc::fence_after_sync();
         const int np = NPJ ? NPJ : jt.n(j) >> 4, ns = (np + 1) >> 1;
@@ -786,11 +789,12 @@ __device__ __forceinline__ void epilogue_scores(const TcArgs& a, const Smem& L, 
             const bool need_mask = t * kTileTok + kTileTok - 1 > s.N - s.W;
             unsigned long long bacc[2] = {0ull, 0ull};
             float qacc = 0.f;
+            const int rot0 = t * (J ? J : jt.n_jobs);
             ok = need_mask
-                     ? score_tile<FASTQ, true, NBUF_LOG2, J, NPJ, WQ>(jt, job, ntile * J, group, tl, b,
-                                                                    k, tok, bacc, qacc)
-                     : score_tile<FASTQ, false, NBUF_LOG2, J, NPJ, WQ>(jt, job, ntile * J, group, tl, b,
-                                                                     k, tok, bacc, qacc);
+                     ? score_tile<FASTQ, true, NBUF_LOG2, J, NPJ, WQ>(jt, job, ntile * J, rot0, group,
+                                                                    tl, b, k, tok, bacc, qacc)
+                     : score_tile<FASTQ, false, NBUF_LOG2, J, NPJ, WQ>(jt, job, ntile * J, rot0, group,
+                                                                     tl, b, k, tok, bacc, qacc);
             if (!ok) break;
             const float2 b2 = tc::unpack2(tc::add2(bacc[0], bacc[1]));
             const float bsum = b2.x + b2.y;

@@ -256,6 +256,48 @@ def test_layer_path_matches_whole_step():
     ctx.close()
 
 
+@pytest.mark.parametrize("name,layers", [("gui", 3), ("qwen-img", 5)])
+def test_layer_path_matches_whole_step_at_paper_shapes(name, layers):
+    """The layer-by-layer calls (score, select, compact) against the whole
+    step, bit for bit, at the paper shapes whose window kernels are compiled
+    as specialised plans (jobs per tile, job sizes and window as constants)."""
+    wl = workloads.CONFIGS[name].with_(layers=layers, requests=1)
+    x = workloads.generate(wl, seed=12, device="cuda")
+    budget = max(wl.budgets)
+    whole = run_gpu(wl, x, budget)
+    p = bacon.default_params(max_seq_len=wl.seq_len, max_requests=1)
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool,
+                        budget, params=p)
+    st = bacon.State(ctx)
+    for l in range(wl.layers):
+        S = st.score_layer(l, x.qwin[0, l], x.k[0, l], scores_out=True)
+        idx = st.select(budget, wl.seq_len)
+        ko, vo = ctx.compact(x.k[0, l], x.v[0, l], idx)
+        ctx.sync()
+        assert np.array_equal(idx.cpu().numpy(), whole["idx"][0, l]), l
+        assert np.array_equal(S.cpu().numpy(), whole["S"][0, l]), l
+        assert torch.equal(ko.cpu(), whole["Kc"][0, l]) and torch.equal(vo.cpu(), whole["Vc"][0, l])
+    st.close()
+    ctx.close()
+
+
+def test_host_path_matches_device_path_at_gui_shape():
+    """bacon_compress_host (page-locked inputs) against the device path, bit
+    for bit, at the GUI shape (specialised window plans) with two layers."""
+    wl = workloads.CONFIGS["gui"].with_(layers=2, requests=2)
+    x = workloads.generate(wl, seed=13, device="cuda")
+    budget = max(wl.budgets)
+    dev = run_gpu(wl, x, budget)
+    p = bacon.default_params(max_seq_len=wl.seq_len, max_requests=2)
+    ctx = bacon.Context(wl.layers, wl.kv_heads, wl.q_heads, wl.head_dim, wl.window, wl.pool,
+                        budget, params=p)
+    qh, kh, vh = (t.cpu().pin_memory() for t in (x.qwin, x.k, x.v))
+    ko, vo, idx = ctx.compress_host(qh, kh, vh, budget)
+    assert np.array_equal(idx.numpy(), dev["idx"])
+    assert torch.equal(ko, dev["Kc"]) and torch.equal(vo, dev["Vc"])
+    ctx.close()
+
+
 @pytest.mark.parametrize("pinned", ["all", "none", "values_pageable"])
 def test_host_path_matches_device_path(pinned):
     """Page-locked values are gathered in place, pageable ones uploaded."""
