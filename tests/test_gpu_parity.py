@@ -654,7 +654,8 @@ def run_with_lse(wl, x, lse, budget):
     return out
 
 
-@pytest.mark.parametrize("name,budget", [("tiny", 64), ("qwen-img", 256), ("gui", 1024)])
+@pytest.mark.parametrize("name,budget", [("tiny", 64), ("qwen-img", 256), ("video", 652),
+                                         ("gui", 1024)])
 def test_prefill_normalisers_path(name, budget):
     """bacon_compress_with_lse (one pass over K) against the oracle at the
     full shape, every unit: the oracle computes its own normalisers in

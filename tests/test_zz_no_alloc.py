@@ -28,6 +28,8 @@ SHAPES = [
                         window=32, visual=(16, 3616))),
     ("gui_layer", dict(layers=1, q_heads=28, kv_heads=4, head_dim=128, seq_len=16384,
                        window=64, visual=(16, 15888))),
+    ("video_layer", dict(layers=1, q_heads=28, kv_heads=4, head_dim=128, seq_len=6528,
+                         window=64, visual=(16, 6288))),
     ("ragged", dict(layers=1, q_heads=6, kv_heads=2, head_dim=128, seq_len=1000, window=5,
                     visual=(16, 900))),
 ]
