@@ -59,6 +59,8 @@ def parse():
 # exponentials per clock per SM of the special-function unit (ex2): the
 # nominal rate of this part (Blackwell Ultra doubles sm_100's 16)
 SFU_EX2_PER_CLK_PER_SM = 32
+# nominal HBM3e bandwidth of this part (GB/s), beside the measured copy rate
+NOMINAL_HBM_GBS = 7900.0
 
 
 def peaks():
@@ -585,6 +587,7 @@ def main():
             "ms_per_request": ms / wl.requests,
             "achieved_step_gbs": step_bytes / (ms / 1e3) / 1e9,
             "step_roofline_frac": step_bytes / (ms / 1e3) / 1e9 / hbm,
+            "step_frac_of_nominal_hbm": step_bytes / (ms / 1e3) / 1e9 / NOMINAL_HBM_GBS,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded, paper-shaped; no datasets)",
             "config": config_dict(wl, budget, world),
