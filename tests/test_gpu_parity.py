@@ -178,6 +178,13 @@ EDGE = [
     # the largest window block the kernels take: G W = 512 rows at d = 128
     ("rows_512_d128", dict(seq_len=1500, layers=2, q_heads=16, kv_heads=2, head_dim=128,
                            window=64, visual=(16, 1400)), 200, {}),
+    # the longest prompt the library takes (24 positions per calibration
+    # thread), and a ragged one just below it with the GQA 7:1, W = 64 window
+    # blocks of the paper's long shapes
+    ("max_prompt", dict(seq_len=24576, layers=2, q_heads=8, kv_heads=2, head_dim=128,
+                        window=32, visual=(16, 24000)), 1024, {}),
+    ("near_max_gqa7", dict(seq_len=24000, layers=2, q_heads=14, kv_heads=2, head_dim=128,
+                           window=64, visual=(16, 23500)), 1024, {}),
 ]
 
 
