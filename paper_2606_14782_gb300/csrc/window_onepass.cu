@@ -241,8 +241,7 @@ __device__ __forceinline__ bool epi_sync(const Bars& b, int& nsync)
 
 // SPEC: the multi-head 1024-token unit (N = 1024, W = 32, 32 window rows)
 // with its sizes as constants: the tile loops unroll and the mask test runs
-// only where a tile can reach into the window (every instruction saved counts:
-// the epilogue is bound by instruction issue).
+// only where a tile can reach into the window.
 template <int D, bool SPEC>
 __device__ void epilogue(const TcArgs& a, const Layout& L, uint8_t* sm, const Bars& b)
 {
