@@ -14,15 +14,16 @@
 // pooling and coherence windows slide along a thread's own positions and
 // the position order of the members is (thread, slot) order: one
 // block-wide exclusive scan gives every thread its tie rank or its output
-// offset.  The per-position arrays in shared memory are stored slot-major,
-// element (slot k, thread t) at k T + t: when every thread of a warp reads
-// its own position plus the same offset, the 32 reads fall in consecutive
-// words (no bank conflicts), and the radix select's passes, which walk the
-// storage index s = k T + t, read consecutive words as well.
+// offset.  The one per-position array in shared memory (the pooled
+// backbone, then the final score: the keys of the two selections) is
+// stored slot-major, element (slot k, thread t) at k T + t, so the radix
+// select's passes, which walk the storage index s = k T + t, read
+// consecutive words, and those are the thread's own slots.  V lives in
+// registers; the windows' neighbours come from global memory.
 //
-// The two standard deviations come from one walk that sums moments about
-// fixed shifts in fp32 (the shifts keep the differences small, so no
-// precision is lost to cancellation).
+// The standard deviations are fp32 sums over the members: B~'s moments
+// about the M-th value (one walk), V's mean and then its squared
+// deviations from it (two walks); neither loses precision to cancellation.
 #include "common.cuh"
 #include "select.cuh"
 
@@ -209,16 +210,129 @@ __device__ __forceinline__ int ties_before(const Slots<T, PER>& arr, int i0, int
     return block_exclusive_scan(eq, warp_sums, total);
 }
 
+// The residual E of the thread's run into x (0 at and past N), added to v
+// when use_E, and the coherence (Eqs. 5-7) with the radius R a constant:
+// v[k] += the mean of E over [i - R, i + R] clipped to [0, N), for the run's
+// positions i = i0 + k < N.  The R values on either side come from the
+// neighbouring lanes' runs by shuffles (from global memory at a warp's two
+// ends, loaded together with the run) and count as 0 outside [0, N).  The
+// window sum slides along the run: drop i - R, add i + 1 + R.  Needs
+// R <= PER and every lane of the warp.
+template <int PER, int R>
+__device__ __forceinline__ void coherence_run(const float* __restrict__ Ec, int i0, int N,
+                                              bool use_E, float* x, float* v)
+{
+    static_assert(R <= PER, "the halo must come from the adjacent run");
+    const int lane = threadIdx.x & 31;
+    load_run<PER>(Ec, i0, N, x);
+    float gl[R], gh[R];
+#pragma unroll
+    for (int m = 0; m < R; ++m) {
+        const int jl = i0 - R + m, jh = i0 + PER + m;
+        gl[m] = (lane == 0 && jl >= 0 && jl < N) ? __ldg(Ec + jl) : 0.f;
+        gh[m] = (lane == 31 && jh < N) ? __ldg(Ec + jh) : 0.f;
+    }
+    if (use_E) {
+#pragma unroll
+        for (int k = 0; k < PER; ++k) v[k] += x[k];
+    }
+    float e[PER + 2 * R];
+#pragma unroll
+    for (int m = 0; m < R; ++m) {
+        const int jl = i0 - R + m, jh = i0 + PER + m;
+        const float lo = __shfl_up_sync(0xffffffffu, x[PER - R + m], 1);
+        const float hi = __shfl_down_sync(0xffffffffu, x[m], 1);
+        e[m] = lane == 0 ? gl[m] : (jl >= 0 ? lo : 0.f);
+        e[R + PER + m] = lane == 31 ? gh[m] : (jh < N ? hi : 0.f);
+    }
+#pragma unroll
+    for (int k = 0; k < PER; ++k) e[R + k] = x[k];
+    const float inv_full = 1.f / (float)(2 * R + 1);  // windows away from the ends
+    float sum = 0.f;
+#pragma unroll
+    for (int j = 0; j <= 2 * R; ++j) sum += e[j];
+#pragma unroll
+    for (int k = 0; k < PER; ++k) {
+        const int i = i0 + k;
+        if (i < N) {
+            const int cnt = min(N - 1, i + R) - max(0, i - R) + 1;
+            float w = inv_full;
+            if (cnt != 2 * R + 1) w = 1.f / (float)cnt;
+            // the window sum of non-negative values: rounding in the slide
+            // can leave ~1e-9 below zero after a large value leaves the
+            // window, so it is clamped
+            v[k] += fmaxf(sum, 0.f) * w;
+        }
+        if (k + 1 < PER) {
+            sum -= e[k];
+            sum += e[k + 2 * R + 1];
+        }
+    }
+}
+
+// The same for any radius, reading the window from global memory (L1).
+template <int PER>
+__device__ __forceinline__ void coherence_any(const float* __restrict__ Ec, int i0, int N, int r,
+                                              float* v)
+{
+    const float inv_full = 1.f / (float)(2 * r + 1);
+    int lo = max(0, i0 - r), hi = min(N - 1, i0 + r);
+    float sum = 0.f;
+    for (int j = lo; j <= hi; ++j) sum += __ldg(Ec + j);
+#pragma unroll
+    for (int k = 0; k < PER; ++k) {
+        const int i = i0 + k;
+        if (i < N) {
+            const int cnt = hi - lo + 1;
+            v[k] += fmaxf(sum, 0.f) * (cnt == 2 * r + 1 ? inv_full : 1.f / (float)cnt);
+            if (i - r >= 0) sum -= __ldg(Ec + i - r);
+            if (i + 1 + r <= N - 1) sum += __ldg(Ec + i + 1 + r);
+            lo = max(0, i + 1 - r);
+            hi = min(N - 1, i + 1 + r);
+        }
+    }
+}
+
+// Whether the run with its halo (PER + 2 R floats) and V (PER floats) fit
+// in the 64 registers a thread has, with room for the rest.
+__host__ __device__ constexpr bool run_fits(int PER, int R) { return R <= PER && 2 * PER + 2 * R <= 56; }
+
+// E (added to v when use_E) and its coherence, with the paper's radii (3, 5,
+// 7, 9) compiled as constants where the registers allow.
+template <int PER>
+__device__ __forceinline__ void residual_and_coherence(const float* __restrict__ Ec, int i0, int N,
+                                                       int r, bool use_E, float* x, float* v)
+{
+    if constexpr (run_fits(PER, 3))
+        if (r == 3) return coherence_run<PER, 3>(Ec, i0, N, use_E, x, v);
+    if constexpr (run_fits(PER, 5))
+        if (r == 5) return coherence_run<PER, 5>(Ec, i0, N, use_E, x, v);
+    if constexpr (run_fits(PER, 7))
+        if (r == 7) return coherence_run<PER, 7>(Ec, i0, N, use_E, x, v);
+    if constexpr (run_fits(PER, 9))
+        if (r == 9) return coherence_run<PER, 9>(Ec, i0, N, use_E, x, v);
+    load_run<PER>(Ec, i0, N, x);
+    if (use_E) {
+#pragma unroll
+        for (int k = 0; k < PER; ++k) v[k] += x[k];
+    }
+    coherence_any<PER>(Ec, i0, N, r, v);
+}
+
 // One unit (request, layer, kv-head) u under hyper-parameters c.  lam_out
 // (may be null) receives lambda; idx_pair is the pair's [Hkv][kept] output.
-// N <= T PER.
+// N <= T PER.  One slot-major array in shared memory holds the pooled
+// backbone and then the final score; V stays in the thread's registers
+// (every later read of it is the thread's own), and the pooling and
+// coherence windows read their neighbours from global memory (L1), so a
+// unit needs T PER floats of shared memory and two CTAs share an SM at the
+// 512-thread classes.
 template <int T, int PER>
 __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, const CalibArgs& a,
                                                int u, float* lam_out, int32_t* idx_pair)
 {
     extern __shared__ __align__(16) float sm[];
-    const Slots<T, PER> A1{sm};            // B (pooling), then E (coherence), then V
-    const Slots<T, PER> A2{sm + T * PER};  // pooled backbone B~, then the final score S
+    const Slots<T, PER> A{sm};  // pooled backbone B~, then the final score S
     // the selections never look at more than T PER keys
     constexpr int kCap = T * PER < kSelCap ? T * PER : kSelCap;
     __shared__ __align__(16) int hist[sel_hist_ints(kCap)];
@@ -248,8 +362,8 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
         const float* Ec = Eof(layer);
         const int nprev = min(c.m, layer);
         const float inv_prev = nprev > 0 ? 1.f / (float)nprev : 0.f;
-        // the residuals are read only after the pooling: start bringing them
-        // into L2 now
+        // the residuals are read only after the pooling and the first
+        // selection: start bringing them into L2 now
         prefetch_l2(Ec, N);
         if (c.use_T)
             for (int j = layer - nprev; j < layer; ++j) prefetch_l2(Eof(j), N);
@@ -257,33 +371,42 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
         // ---- pooled backbone over the candidates (max over [i - half, i + half])
         float x[PER];
         load_run<PER>(Bu, i0, N, x);
-#pragma unroll
-        for (int k = 0; k < PER; ++k) A1.own(k) = x[k];
-        __syncthreads();
         uint32_t kmin = 0xffffffffu, kmax = 0u;  // key range of B~ over the candidates
         const int half = c.pool / 2;
         if (half == 3) {
             // width 7 (the default): the run and three positions either side
-            // in registers, each output a maximum of seven by three max3
-            float w[PER + 6];
+            // in registers (-inf outside the candidates; the neighbours'
+            // values by shuffles, from global memory at a warp's two ends),
+            // each output a maximum of seven by three max3
+            const int lane = threadIdx.x & 31;
+            float hl[3], hr[3];
 #pragma unroll
             for (int m = 0; m < 3; ++m) {
                 const int jl = i0 - 3 + m, jr = i0 + PER + m;
-                w[m] = (jl >= 0 && jl < n_cand) ? A1[jl] : -INFINITY;
-                w[PER + 3 + m] = jr < n_cand ? A1[jr] : -INFINITY;
+                hl[m] = (lane == 0 && jl >= 0 && jl < n_cand) ? __ldg(Bu + jl) : -INFINITY;
+                hr[m] = (lane == 31 && jr < n_cand) ? __ldg(Bu + jr) : -INFINITY;
             }
 #pragma unroll
-            for (int k = 0; k < PER; ++k) w[3 + k] = i0 + k < n_cand ? x[k] : -INFINITY;
+            for (int k = 0; k < PER; ++k)
+                if (i0 + k >= n_cand) x[k] = -INFINITY;
+#pragma unroll
+            for (int m = 0; m < 3; ++m) {
+                const float lo = __shfl_up_sync(0xffffffffu, x[PER - 3 + m], 1);
+                const float hi = __shfl_down_sync(0xffffffffu, x[m], 1);
+                if (lane != 0) hl[m] = lo;
+                if (lane != 31) hr[m] = hi;
+            }
+            auto at = [&](int j) -> float { return j < 0 ? hl[j + 3] : (j >= PER ? hr[j - PER] : x[j]); };
 #pragma unroll
             for (int k = 0; k < PER; ++k) {
                 float mx = 0.f;
                 if (i0 + k < n_cand) {
-                    mx = max3f(max3f(w[k], w[k + 1], w[k + 2]),
-                                 max3f(w[k + 3], w[k + 4], w[k + 5]), w[k + 6]);
+                    mx = max3f(max3f(at(k - 3), at(k - 2), at(k - 1)),
+                               max3f(at(k), at(k + 1), at(k + 2)), at(k + 3));
                     kmin = min(kmin, float_key(mx));
                     kmax = max(kmax, float_key(mx));
                 }
-                A2.own(k) = mx;
+                A.own(k) = mx;
             }
         } else {
 #pragma unroll
@@ -293,12 +416,32 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
                 if (i < n_cand) {
                     mx = -INFINITY;
                     const int lo = max(0, i - half), hi = min(n_cand - 1, i + half);
-                    for (int v = lo; v <= hi; ++v) mx = fmaxf(mx, A1[v]);
+                    for (int v = lo; v <= hi; ++v) mx = fmaxf(mx, __ldg(Bu + v));
                     kmin = min(kmin, float_key(mx));
                     kmax = max(kmax, float_key(mx));
                 }
-                A2.own(k) = mx;
+                A.own(k) = mx;
             }
+        }
+        if (a.Bp) {
+#pragma unroll
+            for (int k = 0; k < PER; ++k) x[k] = A.own(k);
+            store_run<PER>(a.Bp + (size_t)u * N, i0, N, x);
+        }
+
+        // ---- the M best candidates by B~ (Eq. 12); V is computed after this
+        // selection, so that it is not held across it
+        const int calib_keep = min(a.calib_budget[pair], N) - win;
+        const long long Ml = (long long)c.rho * (long long)(calib_keep > 0 ? calib_keep : 0);
+        const int M = (int)(Ml < n_cand ? Ml : n_cand);
+        uint32_t mem = 0u;
+        float pb = 0.f;
+        if (M > 0) {
+            const SelectResult sel = radix_select_range<kCap>(T * PER, M, SlotKeys<T, PER>{A.a, n_cand},
+                                                        hist, bcast, kmin, kmax);
+            const int eqb = ties_before(A, i0, n_cand, sel, warp_sums, &total_s);
+            mem = members(A, i0, n_cand, sel, eqb);
+            pb = key_float(sel.tau);
         }
 
         // ---- persistence: mean of E over the preceding min(m, l) layers (Eqs. 8-9)
@@ -306,99 +449,65 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
 #pragma unroll
         for (int k = 0; k < PER; ++k) v[k] = 0.f;
         if (c.use_T) {
+            // a layer's run in chunks of at most 16 (V and one chunk in
+            // registers)
+            constexpr int CH = PER <= 16 ? PER : PER / 2;
+            static_assert(PER % CH == 0 && CH % 4 == 0, "chunks of whole 16-byte loads");
             for (int j = layer - nprev; j < layer; ++j) {
-                float e[PER];
-                load_run<PER>(Eof(j), i0, N, e);
 #pragma unroll
-                for (int k = 0; k < PER; ++k) v[k] += e[k];
+                for (int c0 = 0; c0 < PER; c0 += CH) {
+                    float e[CH];
+                    load_run<CH>(Eof(j), i0 + c0, N, e);
+#pragma unroll
+                    for (int k = 0; k < CH; ++k) v[c0 + k] += e[k];
+                }
             }
 #pragma unroll
             for (int k = 0; k < PER; ++k) v[k] *= inv_prev;
         }
-        __syncthreads();  // every pooling read of A1 is done
-        load_run<PER>(Ec, i0, N, x);
-#pragma unroll
-        for (int k = 0; k < PER; ++k) {
-            A1.own(k) = x[k];
-            if (c.use_E) v[k] += x[k];
-        }
-        __syncthreads();
-        // ---- coherence: truncated radius-r box mean of E (Eqs. 5-7), the
-        // window sum sliding along the run
+        // ---- E, and the coherence: truncated radius-r box mean of E (Eqs. 5-7)
         if (c.use_L) {
-            const int r = c.r;
-            const float inv_full = 1.f / (float)(2 * r + 1);  // windows away from the ends
-            int lo = max(0, i0 - r), hi = min(N - 1, i0 + r);
-            float sum = 0.f;
-            for (int j = lo; j <= hi; ++j) sum += A1[j];
+            residual_and_coherence<PER>(Ec, i0, N, c.r, c.use_E, x, v);
+        } else if (c.use_E) {
+            load_run<PER>(Ec, i0, N, x);
 #pragma unroll
-            for (int k = 0; k < PER; ++k) {
-                const int i = i0 + k;
-                if (i < N) {
-                    // the window sum of non-negative values: rounding in the
-                    // slide can leave ~1e-9 below zero after a large value
-                    // leaves the window, so it is clamped
-                    const int cnt = hi - lo + 1;
-                    v[k] += fmaxf(sum, 0.f) * (cnt == 2 * r + 1 ? inv_full : 1.f / (float)cnt);
-                    // the window of i + 1: drop i - r, add i + 1 + r
-                    if (i - r >= 0) sum -= A1[i - r];
-                    if (i + 1 + r <= N - 1) sum += A1[i + 1 + r];
-                    lo = max(0, i + 1 - r);
-                    hi = min(N - 1, i + 1 + r);
-                }
-            }
+            for (int k = 0; k < PER; ++k) v[k] += x[k];
         }
-        float vsum = 0.f;  // over the candidates: the shift of the moments below
 #pragma unroll
-        for (int k = 0; k < PER; ++k) {
+        for (int k = 0; k < PER; ++k)
             if (i0 + k >= N) v[k] = 0.f;
-            if (i0 + k < n_cand) vsum += v[k];
-        }
         if (a.V) store_run<PER>(a.V + (size_t)u * N, i0, N, v);
-        // V moves to the E array (own slots) for the rest of the unit: it
-        // is read only by its own thread from here on
-        __syncthreads();  // every coherence read of A1 is done
-#pragma unroll
-        for (int k = 0; k < PER; ++k) A1.own(k) = v[k];
-        if (a.Bp) {
-#pragma unroll
-            for (int k = 0; k < PER; ++k) x[k] = A2.own(k);
-            store_run<PER>(a.Bp + (size_t)u * N, i0, N, x);
-        }
 
-        // ---- Eqs. 12-15
-        const int calib_keep = min(a.calib_budget[pair], N) - win;
-        const long long Ml = (long long)c.rho * (long long)(calib_keep > 0 ? calib_keep : 0);
-        const int M = (int)(Ml < n_cand ? Ml : n_cand);
+        // ---- lambda over the M members (Eqs. 13-15).  B~ by moments about
+        // the M-th value (every member is at or above it, so the fp32
+        // differences stay small); V by its members' mean, then the mean
+        // square deviation from it (two reductions).
         float lam = 0.f;
         if (M > 0) {
-            // (the candidates' V sum rides on the selection's first reduction)
-            float vtot = 0.f;
-            const SelectResult sel = radix_select_range<kCap>(T * PER, M, SlotKeys<T, PER>{A2.a, n_cand},
-                                                        hist, bcast, kmin, kmax, vsum, &vtot);
-            const int eqb = ties_before(A2, i0, n_cand, sel, warp_sums, &total_s);
-            const uint32_t mem = members(A2, i0, n_cand, sel, eqb);
-            // moments about fixed shifts in one walk: B~ about its M-th value,
-            // V about its mean over the candidates (both near the members'
-            // means, so the fp32 differences keep their precision)
-            const float pb = key_float(sel.tau);
-            const float pv = vtot / (float)n_cand;
             float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
             for (int k = 0; k < PER; ++k) {
                 if ((mem >> k) & 1u) {
-                    const float db = A2.own(k) - pb, dv = A1.own(k) - pv;
+                    const float db = A.own(k) - pb;
                     acc.x += db;
                     acc.y = fmaf(db, db, acc.y);
-                    acc.z += dv;
-                    acc.w = fmaf(dv, dv, acc.w);
+                    acc.z += v[k];
                 }
             }
             const float4 tot = block_sum4(acc, red);
             const float inv_m = 1.f / (float)M;
             const float mb = tot.x * inv_m, mv = tot.z * inv_m;
+            float4 dev = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int k = 0; k < PER; ++k) {
+                if ((mem >> k) & 1u) {
+                    const float dv = v[k] - mv;
+                    dev.x = fmaf(dv, dv, dev.x);
+                }
+            }
+            const float varv = block_sum4(dev, red).x * inv_m;
             const float stdb = sqrtf(fmaxf(tot.y * inv_m - mb * mb, 0.f));
-            const float stdv = sqrtf(fmaxf(tot.w * inv_m - mv * mv, 0.f));
+            const float stdv = sqrtf(varv);
             lam = c.gamma * stdb / (stdv + c.eps);
         }
         if (threadIdx.x == 0 && lam_out) *lam_out = lam;
@@ -407,11 +516,11 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
         for (int k = 0; k < PER; ++k) {
             float sv = 0.f;
             if (i0 + k < n_cand) {
-                sv = fmaf(lam, A1.own(k), A2.own(k));
+                sv = fmaf(lam, v[k], A.own(k));
                 skmin = min(skmin, float_key(sv));
                 skmax = max(skmax, float_key(sv));
             }
-            A2.own(k) = sv;
+            A.own(k) = sv;
             x[k] = sv;
         }
         if (a.write_S) store_run<PER>(a.S + (size_t)u * N, i0, N, x);
@@ -421,7 +530,7 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
         load_run<PER>(a.S + (size_t)u * N, i0, N, x);
 #pragma unroll
         for (int k = 0; k < PER; ++k) {
-            A2.own(k) = x[k];
+            A.own(k) = x[k];
             if (i0 + k < n_cand) {
                 skmin = min(skmin, float_key(x[k]));
                 skmax = max(skmax, float_key(x[k]));
@@ -436,10 +545,10 @@ __device__ __forceinline__ void calibrate_unit(const Shape& s, const Calib& c, c
     if (keep >= n_cand) {
         for (int i = threadIdx.x; i < n_cand; i += blockDim.x) out[i] = i;
     } else if (keep > 0) {
-        const SelectResult sel = radix_select_range<kCap>(T * PER, keep, SlotKeys<T, PER>{A2.a, n_cand},
+        const SelectResult sel = radix_select_range<kCap>(T * PER, keep, SlotKeys<T, PER>{A.a, n_cand},
                                                     hist, bcast, skmin, skmax);
-        const int eqb = ties_before(A2, i0, n_cand, sel, warp_sums, &total_s);
-        const uint32_t mem = members(A2, i0, n_cand, sel, eqb);
+        const int eqb = ties_before(A, i0, n_cand, sel, warp_sums, &total_s);
+        const uint32_t mem = members(A, i0, n_cand, sel, eqb);
         int pos = block_exclusive_scan(__popc(mem), warp_sums, &total_s);
 #pragma unroll
         for (int k = 0; k < PER; ++k)
@@ -474,7 +583,7 @@ calibrate_sweep_kernel(Shape s, CalibTable t, CalibArgs a)
 template <int T, int PER>
 constexpr size_t smem_bytes()
 {
-    return (size_t)2 * T * PER * sizeof(float);
+    return (size_t)T * PER * sizeof(float);
 }
 
 template <int T, int PER>
@@ -513,16 +622,6 @@ cudaError_t by_size(int N, F f)
     return cudaErrorInvalidValue;
 }
 
-struct SmemOf {
-    size_t* out;
-    template <int T, int PER>
-    cudaError_t run() const
-    {
-        *out = smem_bytes<T, PER>();
-        return cudaSuccess;
-    }
-};
-
 struct SelectLaunch {
     const Shape& s;
     const Calib& c;
@@ -543,13 +642,6 @@ struct SweepLaunch {
 };
 
 }  // namespace
-
-size_t calibrate_smem(int N)
-{
-    size_t bytes = 0;
-    by_size(N, SmemOf{&bytes});
-    return bytes;
-}
 
 cudaError_t launch_calibrate_select(const Shape& s, const Calib& c, const CalibArgs& a,
                                     cudaStream_t st)

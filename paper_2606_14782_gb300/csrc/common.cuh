@@ -112,9 +112,6 @@ struct CalibTable {
 cudaError_t launch_calibrate_sweep(const Shape& s, const CalibTable& t, int variants,
                                    const CalibArgs& a, cudaStream_t st);
 
-// Dynamic shared memory of the calibration kernel for N tokens.
-size_t calibrate_smem(int N);
-
 // AdaKV-style selection over the heads of each (request, layer).
 struct AdaptArgs {
     const float* S;              // [units][N] final scores (0 off-candidates)
