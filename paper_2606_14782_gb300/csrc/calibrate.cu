@@ -19,7 +19,8 @@
 // stored slot-major, element (slot k, thread t) at k T + t, so the radix
 // select's passes, which walk the storage index s = k T + t, read
 // consecutive words, and those are the thread's own slots.  V lives in
-// registers; the windows' neighbours come from global memory.
+// registers; the windows' neighbours come from the adjacent lanes' runs by
+// warp shuffles (from global memory at a warp's two ends).
 //
 // The standard deviations are fp32 sums over the members: B~'s moments
 // about the M-th value (one walk), V's mean and then its squared
